@@ -1,0 +1,404 @@
+/*
+ * specflash_oracle.c -- plain, slow, fp64 CPU oracle for the SpecFLASH
+ * target-model verification step (arXiv 2505.12728).
+ *
+ * TEST INFRASTRUCTURE ONLY.  This file is the correctness reference that the
+ * CUDA path is compared against.  Only the test suite, the smoke check and the
+ * CPU-baseline leg of the benchmark may load it.  The product library never
+ * links, loads or calls it, and it shares no code, header, table or helper
+ * with the CUDA path.
+ *
+ * What it computes (all arithmetic in double precision):
+ *
+ *   1. Verification attention (Sec. 3.1, "Preliminaries": the target model
+ *      scores the K candidate tokens in parallel in a single forward pass
+ *      against its cache of visual-then-text tokens).  For every sequence b,
+ *      new query row i < n_q and query head h, with KV head h / (H_q / H_kv):
+ *      the visible keys are the L_b prefix tokens plus draft rows 0..i
+ *      (causal inside the draft block), s_t = scale * <q, k_t>,
+ *      lse = log sum_t exp(s_t), o = sum_t exp(s_t - lse) v_t.
+ *      This is the plain definition; no blocking, no online softmax.
+ *
+ *   2. Decode attention: one query against T contiguous keys.  A separate,
+ *      independently written routine, so that "a k-row verify equals k
+ *      sequential decodes" (the K = 1 degenerate case of the ablation on the
+ *      draft length K) can be checked.
+ *
+ *   3. Acceptance (Sec. 3.1 and Sec. 3.3, the token-wise acceptance-rejection
+ *      rule of the speculative-sampling method the paper cites): per sequence,
+ *      candidate T'_{i+1} is accepted with probability min(1, p_i(x)/q_i(x)),
+ *      the candidates are examined in order up to the first rejection j, and
+ *      the token at position j is drawn from the residual distribution
+ *      norm(max(0, p_j - q_j)), or from the bonus row p_k when all K drafts
+ *      were accepted.  At temperature 0 (greedy decoding, Sec. 4.2) a draft is
+ *      accepted iff it equals the argmax of the target logits.
+ *
+ * Readings of points the paper leaves open (each one is listed with its
+ * reason in the design notes of the repository):
+ *   - acceptance test: u * q(x) < p(x) with a strict "<" (u in [0,1));
+ *   - greedy argmax ties go to the lowest token id; the argmax is taken on
+ *     the raw fp32 logits;
+ *   - all K accepted: a bonus token is drawn from row K of the target logits;
+ *   - uniforms: u_0..u_{K-1} for the K tests, u_K for the single final draw;
+ *   - residual with zero mass (rounding only): draw from p_j instead;
+ *   - inverse CDF in ascending token id: the smallest x with u*S < C(x); if
+ *     rounding leaves none, the last x with non-zero mass;
+ *   - temperature: p = softmax(logits / tau); q is used as given;
+ *   - scores are scaled by `scale` (1/sqrt(d) unless given); the LSE is the
+ *     natural log of the sum of exp of the scaled scores.
+ *
+ * Every function here is pinned by the not-gpu tests against closed forms,
+ * library routines, brute force and the distributional guarantee of the
+ * acceptance rule; none is "parity unpinned".
+ */
+#include <math.h>
+#include <stdint.h>
+#include <stdlib.h>
+#include <string.h>
+
+#define ORACLE_OK 0
+#define ORACLE_ERR_ARG 1
+#define ORACLE_ERR_BAD_PAGE 2
+#define ORACLE_ERR_BAD_TOKEN 3
+#define ORACLE_ERR_NOMEM 4
+
+/* bf16 is the upper half of an IEEE binary32; widening is exact. */
+static double oracle_bf16_value(uint16_t bits)
+{
+    uint32_t w = ((uint32_t)bits) << 16;
+    float f;
+    memcpy(&f, &w, sizeof f);
+    return (double)f;
+}
+
+/* ------------------------------------------------------------------------ */
+/* Decode attention: one query row q[d] against keys k[T][d], values v[T][d]. */
+/* ------------------------------------------------------------------------ */
+int oracle_decode_attention(const double *q, const double *k, const double *v,
+                            int T, int d, double scale, double *o,
+                            double *lse_out)
+{
+    if (T <= 0 || d <= 0 || !q || !k || !v || !o)
+        return ORACLE_ERR_ARG;
+    double *s = (double *)malloc(sizeof(double) * (size_t)T);
+    if (!s)
+        return ORACLE_ERR_NOMEM;
+
+    double smax = -INFINITY;
+    for (int t = 0; t < T; ++t) {
+        double acc = 0.0;
+        for (int c = 0; c < d; ++c)
+            acc += q[c] * k[(size_t)t * d + c];
+        s[t] = scale * acc;
+        if (s[t] > smax)
+            smax = s[t];
+    }
+    double z = 0.0;
+    for (int t = 0; t < T; ++t)
+        z += exp(s[t] - smax);
+    double lse = smax + log(z);
+
+    for (int c = 0; c < d; ++c)
+        o[c] = 0.0;
+    for (int t = 0; t < T; ++t) {
+        double w = exp(s[t] - lse);
+        for (int c = 0; c < d; ++c)
+            o[c] += w * v[(size_t)t * d + c];
+    }
+    if (lse_out)
+        *lse_out = lse;
+    free(s);
+    return ORACLE_OK;
+}
+
+/* ------------------------------------------------------------------------ */
+/* Verification attention over a paged cache.                               */
+/*                                                                          */
+/* q        bf16 bits [B][n_q][H_q][d]                                      */
+/* k_cache  bf16 bits [num_pages][H_kv][page_size][d]   (v_cache the same)  */
+/* block_table [B][max_pages_per_seq]: logical page -> physical page        */
+/* seq_lens [B]: L_b + n_q (the draft rows' K/V are already in the cache)   */
+/* out [B][n_q][H_q][d], lse [B][n_q][H_q] (lse may be NULL)                */
+/*                                                                          */
+/* Only the rows selected by (b_sel, i_sel, h_sel) are computed when those   */
+/* are >= 0 (a negative selector means "all"), so that full-size workloads  */
+/* can be checked on sampled rows.                                          */
+/* ------------------------------------------------------------------------ */
+static int oracle_verify_one_row(const uint16_t *q, const uint16_t *k_cache,
+                                 const uint16_t *v_cache,
+                                 const int32_t *block_table,
+                                 const int32_t *seq_lens, int b, int i, int h,
+                                 int n_q, int H_q, int H_kv, int d,
+                                 int page_size, int num_pages,
+                                 int max_pages_per_seq, double scale,
+                                 double *out, double *lse)
+{
+    const int group = H_q / H_kv;
+    const int h_kv = h / group;
+    const int T = seq_lens[b];
+    const int L = T - n_q;          /* prefix length before the draft block */
+    const int visible = L + i + 1;  /* prefix + draft rows 0..i            */
+
+    const uint16_t *qrow = q + (((size_t)b * n_q + i) * H_q + h) * d;
+    double *s = (double *)malloc(sizeof(double) * (size_t)visible);
+    if (!s)
+        return ORACLE_ERR_NOMEM;
+
+    /* scores */
+    double smax = -INFINITY;
+    for (int t = 0; t < visible; ++t) {
+        int logical_page = t / page_size;
+        int slot = t % page_size;
+        int page = block_table[(size_t)b * max_pages_per_seq + logical_page];
+        if (page < 0 || page >= num_pages) {
+            free(s);
+            return ORACLE_ERR_BAD_PAGE;
+        }
+        const uint16_t *krow =
+            k_cache + (((size_t)page * H_kv + h_kv) * page_size + slot) * d;
+        double acc = 0.0;
+        for (int c = 0; c < d; ++c)
+            acc += oracle_bf16_value(qrow[c]) * oracle_bf16_value(krow[c]);
+        s[t] = scale * acc;
+        if (s[t] > smax)
+            smax = s[t];
+    }
+    double z = 0.0;
+    for (int t = 0; t < visible; ++t)
+        z += exp(s[t] - smax);
+    const double row_lse = smax + log(z);
+
+    double *orow = out + (((size_t)b * n_q + i) * H_q + h) * d;
+    for (int c = 0; c < d; ++c)
+        orow[c] = 0.0;
+    for (int t = 0; t < visible; ++t) {
+        int page = block_table[(size_t)b * max_pages_per_seq + t / page_size];
+        const uint16_t *vrow =
+            v_cache +
+            (((size_t)page * H_kv + h_kv) * page_size + (t % page_size)) * d;
+        double w = exp(s[t] - row_lse);
+        for (int c = 0; c < d; ++c)
+            orow[c] += w * oracle_bf16_value(vrow[c]);
+    }
+    if (lse)
+        lse[((size_t)b * n_q + i) * H_q + h] = row_lse;
+    free(s);
+    return ORACLE_OK;
+}
+
+int oracle_verify_attention(const uint16_t *q, const uint16_t *k_cache,
+                            const uint16_t *v_cache, const int32_t *block_table,
+                            const int32_t *seq_lens, int B, int n_q, int H_q,
+                            int H_kv, int d, int page_size, int num_pages,
+                            int max_pages_per_seq, double scale, int b_sel,
+                            int i_sel, int h_sel, double *out, double *lse)
+{
+    if (!q || !k_cache || !v_cache || !block_table || !seq_lens || !out)
+        return ORACLE_ERR_ARG;
+    if (B <= 0 || n_q <= 0 || H_q <= 0 || H_kv <= 0 || d <= 0 ||
+        page_size <= 0 || num_pages <= 0 || max_pages_per_seq <= 0)
+        return ORACLE_ERR_ARG;
+    if (H_q % H_kv != 0)
+        return ORACLE_ERR_ARG;
+    for (int b = 0; b < B; ++b) {
+        if (seq_lens[b] < n_q ||
+            seq_lens[b] > (long long)max_pages_per_seq * page_size)
+            return ORACLE_ERR_ARG;
+    }
+    if (scale == 0.0)
+        scale = 1.0 / sqrt((double)d);
+
+    int status = ORACLE_OK;
+    const long long rows = (long long)B * n_q * H_q;
+#pragma omp parallel for schedule(dynamic, 1)
+    for (long long r = 0; r < rows; ++r) {
+        int h = (int)(r % H_q);
+        int i = (int)((r / H_q) % n_q);
+        int b = (int)(r / ((long long)H_q * n_q));
+        if ((b_sel >= 0 && b != b_sel) || (i_sel >= 0 && i != i_sel) ||
+            (h_sel >= 0 && h != h_sel))
+            continue;
+        int st = oracle_verify_one_row(q, k_cache, v_cache, block_table,
+                                       seq_lens, b, i, h, n_q, H_q, H_kv, d,
+                                       page_size, num_pages, max_pages_per_seq,
+                                       scale, out, lse);
+        if (st != ORACLE_OK) {
+#pragma omp critical
+            status = st;
+        }
+    }
+    return status;
+}
+
+/* ------------------------------------------------------------------------ */
+/* Target distribution of one verified position: p = softmax(logits / tau).  */
+/* ------------------------------------------------------------------------ */
+int oracle_target_probs(const float *logits, int V, double tau, double *p)
+{
+    if (!logits || !p || V <= 0 || !(tau > 0.0))
+        return ORACLE_ERR_ARG;
+    double zmax = -INFINITY;
+    for (int x = 0; x < V; ++x) {
+        double z = (double)logits[x] / tau;
+        if (z > zmax)
+            zmax = z;
+    }
+    double sum = 0.0;
+    for (int x = 0; x < V; ++x) {
+        p[x] = exp((double)logits[x] / tau - zmax);
+        sum += p[x];
+    }
+    for (int x = 0; x < V; ++x)
+        p[x] /= sum;
+    return ORACLE_OK;
+}
+
+/* Greedy decoding's choice: the first index holding the largest logit. */
+int oracle_argmax(const float *logits, int V)
+{
+    int best = 0;
+    for (int x = 1; x < V; ++x)
+        if (logits[x] > logits[best])
+            best = x;
+    return best;
+}
+
+/* ------------------------------------------------------------------------ */
+/* Acceptance for a batch of sequences.                                     */
+/*                                                                          */
+/* target_logits [B][k+1][V] fp32: row i scores draft i, row k is the bonus */
+/* draft_probs   [B][k][V]   fp32: q_i, used as given                        */
+/* draft_tokens  [B][k]      int32: T'_1..T'_k                              */
+/* uniforms      [B][k+1]    fp32 in [0,1)                                  */
+/* temperature   [B]         fp32: <= 0 means greedy for that sequence       */
+/* outputs: num_accepted [B]; out_tokens [B][k+1] (first num_accepted + 1    */
+/* valid, the rest -1); accept_ratio [B][k] = min(1, p/q) (greedy: 1 or 0),  */
+/* may be NULL; margin [B][k+1] (may be NULL): for each test actually       */
+/* evaluated |u_i - p/q| (q = 0: +inf), for the final draw the distance of  */
+/* u_k to the nearest normalised CDF boundary; +inf where no floating-point */
+/* comparison decides the outcome.                                          */
+/* ------------------------------------------------------------------------ */
+int oracle_accept(const float *target_logits, const float *draft_probs,
+                  const int32_t *draft_tokens, const float *uniforms,
+                  const float *temperature, int B, int k, int V,
+                  int32_t *num_accepted, int32_t *out_tokens,
+                  double *accept_ratio, double *margin)
+{
+    if (!target_logits || !draft_probs || !draft_tokens || !uniforms ||
+        !temperature || !num_accepted || !out_tokens)
+        return ORACLE_ERR_ARG;
+    if (B <= 0 || k <= 0 || V <= 0)
+        return ORACLE_ERR_ARG;
+    for (long long n = 0; n < (long long)B * k; ++n)
+        if (draft_tokens[n] < 0 || draft_tokens[n] >= V)
+            return ORACLE_ERR_BAD_TOKEN;
+
+    double *p = (double *)malloc(sizeof(double) * (size_t)V);
+    double *r = (double *)malloc(sizeof(double) * (size_t)V);
+    if (!p || !r) {
+        free(p);
+        free(r);
+        return ORACLE_ERR_NOMEM;
+    }
+
+    for (int b = 0; b < B; ++b) {
+        const float tau = temperature[b];
+        const int greedy = !(tau > 0.0f);
+        const float *rows = target_logits + (size_t)b * (k + 1) * V;
+        const float *qrows = draft_probs + (size_t)b * k * V;
+        const int32_t *x = draft_tokens + (size_t)b * k;
+        const float *u = uniforms + (size_t)b * (k + 1);
+        double *mg = margin ? margin + (size_t)b * (k + 1) : NULL;
+        if (mg)
+            for (int i = 0; i <= k; ++i)
+                mg[i] = INFINITY;
+
+        /* Score every draft (the target computes all rows in one pass), and
+         * take the decisions in order up to the first rejection j. */
+        int j = k;
+        for (int i = 0; i < k; ++i) {
+            const float *row = rows + (size_t)i * V;
+            int accept;
+            double ratio;
+            double m = INFINITY;
+            if (greedy) {
+                accept = (x[i] == oracle_argmax(row, V));
+                ratio = accept ? 1.0 : 0.0;
+            } else {
+                oracle_target_probs(row, V, (double)tau, p);
+                double pt = p[x[i]];
+                double qt = (double)qrows[(size_t)i * V + x[i]];
+                accept = ((double)u[i] * qt < pt);
+                if (qt > 0.0) {
+                    ratio = pt / qt < 1.0 ? pt / qt : 1.0;
+                    m = fabs((double)u[i] - pt / qt);
+                } else {
+                    ratio = 1.0;
+                }
+            }
+            if (accept_ratio)
+                accept_ratio[(size_t)b * k + i] = ratio;
+            if (j == k) {
+                if (mg)
+                    mg[i] = m;
+                if (!accept)
+                    j = i;
+            }
+        }
+
+        /* The token at position j: corrected (j < k) or bonus (j == k). */
+        int final_token;
+        const float *row_j = rows + (size_t)j * V;
+        if (greedy) {
+            final_token = oracle_argmax(row_j, V);
+        } else {
+            oracle_target_probs(row_j, V, (double)tau, p);
+            double mass = 0.0;
+            if (j < k) {
+                const float *qj = qrows + (size_t)j * V;
+                for (int y = 0; y < V; ++y) {
+                    double diff = p[y] - (double)qj[y];
+                    r[y] = diff > 0.0 ? diff : 0.0;
+                    mass += r[y];
+                }
+            }
+            if (j == k || !(mass > 0.0)) {
+                mass = 0.0;
+                for (int y = 0; y < V; ++y) {
+                    r[y] = p[y];
+                    mass += r[y];
+                }
+            }
+            const double target = (double)u[k] * mass;
+            double cdf = 0.0;
+            double nearest = INFINITY;
+            final_token = -1;
+            int last_positive = -1;
+            for (int y = 0; y < V; ++y) {
+                cdf += r[y];
+                if (r[y] > 0.0)
+                    last_positive = y;
+                double dist = fabs((double)u[k] - cdf / mass);
+                if (dist < nearest)
+                    nearest = dist;
+                if (final_token < 0 && target < cdf)
+                    final_token = y;
+            }
+            if (final_token < 0)
+                final_token = last_positive;
+            if (mg)
+                mg[k] = nearest;
+        }
+
+        num_accepted[b] = j;
+        int32_t *ob = out_tokens + (size_t)b * (k + 1);
+        for (int i = 0; i <= k; ++i)
+            ob[i] = -1;
+        for (int i = 0; i < j; ++i)
+            ob[i] = x[i];
+        ob[j] = final_token;
+    }
+    free(p);
+    free(r);
+    return ORACLE_OK;
+}

@@ -1,0 +1,72 @@
+"""The oracle's pins must reject plausible mistakes.
+
+Each case plants one mistake in a copy of the oracle's C source (on the CPU,
+in a temporary directory), compiles it, and runs the oracle pin tests against
+the broken copy.  The pins pass on the real oracle (the other test files) and
+must fail on every mutant here; a mutant that survives means a pin is missing.
+"""
+import os
+import subprocess
+import sys
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+SRC = os.path.join(ROOT, "oracle", "specflash_oracle.c")
+
+MUTANTS = {
+    "accept_test_flipped": ("accept = ((double)u[i] * qt < pt);",
+                            "accept = ((double)u[i] * qt > pt);"),
+    "residual_q_minus_p": ("double diff = p[y] - (double)qj[y];",
+                           "double diff = (double)qj[y] - p[y];"),
+    "residual_not_normalised": ("const double target = (double)u[k] * mass;",
+                                "const double target = (double)u[k];"),
+    "final_draw_from_next_row": ("const float *row_j = rows + (size_t)j * V;",
+                                 "const float *row_j = rows + (size_t)(j < k ? j + 1 : j) * V;"),
+    "final_draw_reuses_test_uniform": ("const double target = (double)u[k] * mass;",
+                                       "const double target = (double)u[j] * mass;"),
+    "greedy_last_maximum": ("if (logits[x] > logits[best])",
+                            "if (logits[x] >= logits[best])"),
+    "temperature_ignored": [("double z = (double)logits[x] / tau;",
+                             "double z = (double)logits[x];"),
+                            ("p[x] = exp((double)logits[x] / tau - zmax);",
+                             "p[x] = exp((double)logits[x] - zmax);")],
+    "decisions_past_first_rejection": ("            if (j == k) {\n                if (mg)",
+                                       "            {\n                if (mg)"),
+    "no_causal_mask": ("const int visible = L + i + 1;", "const int visible = T;"),
+    "causal_off_by_one": ("const int visible = L + i + 1;", "const int visible = L + i + (i > 0);"),
+    "gqa_modulo_mapping": ("const int h_kv = h / group;", "const int h_kv = h % H_kv;"),
+    "scale_dropped": ("        s[t] = scale * acc;\n        if (s[t] > smax)\n            smax = s[t];\n    }\n    double z = 0.0;\n    for (int t = 0; t < visible; ++t)",
+                      "        s[t] = acc;\n        if (s[t] > smax)\n            smax = s[t];\n    }\n    double z = 0.0;\n    for (int t = 0; t < visible; ++t)"),
+    "slot_shifted": ("int slot = t % page_size;", "int slot = (t + 1) % page_size;"),
+    "values_read_from_keys": ("        const uint16_t *vrow =\n            v_cache +",
+                              "        const uint16_t *vrow =\n            k_cache +"),
+}
+
+
+@pytest.fixture(scope="module")
+def source():
+    with open(SRC) as f:
+        return f.read()
+
+
+@pytest.mark.parametrize("name", sorted(MUTANTS))
+def test_pins_reject_mutant(name, source, tmp_path):
+    edits = MUTANTS[name]
+    edits = edits if isinstance(edits, list) else [edits]
+    mutated = source
+    for find, repl in edits:
+        assert mutated.count(find) == 1, f"mutation anchor for {name} not unique"
+        mutated = mutated.replace(find, repl)
+    c_path = tmp_path / "mutant.c"
+    so_path = tmp_path / "libmutant.so"
+    c_path.write_text(mutated)
+    subprocess.run(["gcc", "-O2", "-std=c11", "-fPIC", "-shared", "-fopenmp", str(c_path),
+                    "-o", str(so_path), "-lm"], check=True)
+    env = dict(os.environ, SPECFLASH_ORACLE_LIB=str(so_path))
+    proc = subprocess.run(
+        [sys.executable, "-m", "pytest", "-x", "-q", "-p", "no:cacheprovider",
+         os.path.join(ROOT, "tests", "test_oracle_attention.py"),
+         os.path.join(ROOT, "tests", "test_oracle_accept.py")],
+        cwd=ROOT, env=env, capture_output=True, text=True, timeout=600)
+    assert proc.returncode != 0, f"mutant {name} survived the oracle pins:\n{proc.stdout[-2000:]}"
