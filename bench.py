@@ -1,0 +1,434 @@
+"""Benchmark of the SpecFLASH verification step on GB300.
+
+One step = one pass of the whole hot path over one batch: verification
+attention for every layer of the workload (one sf_verify_attention call per
+layer, separate KV caches) followed by the acceptance rule (sf_accept).
+Default workload: the image-LMM 7B shape (B1, 32 layers, 32/32 heads, d128,
+prefix 3008 = 5x576 visual + 128 text, k=5 drafts, V=32000, sampling at
+tau=1): 1.58 GB of KV per step, far larger than the 129 MB L2, so every step
+streams the caches from HBM.
+
+Prints ONE JSON line (rank 0).  `value` is draft tokens verified per second
+over the whole job; `e2e` repeats the measurement through host buffers
+(pinned host -> device copies of the step's inputs and a device -> host read
+of its results inside the timed region).
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME]
+  python bench.py --impl reference ...   # the CPU oracle, same metric
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = ("verify-step latency (µs) and KV-cache HBM GB/s vs GB300 peak; "
+          "draft tokens verified/sec")
+UNIT = "draft tokens/s"
+NOMINAL_HBM_GBS = 8000.0
+
+
+# --------------------------------------------------------------------------- #
+# distributed plumbing (one process per GPU, launched by torchrun)            #
+# --------------------------------------------------------------------------- #
+def dist_env():
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return rank, world, local
+
+
+def init_dist(world: int, backend: str):
+    import torch.distributed as dist
+    if world > 1 and not dist.is_initialized():
+        dist.init_process_group(backend=backend)
+    return dist
+
+
+def barrier(world: int):
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+def max_over_ranks(x: float, world: int, device=None) -> float:
+    """Largest value of x across ranks (the job is as slow as its slowest rank)."""
+    if world <= 1:
+        return float(x)
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([float(x)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+# --------------------------------------------------------------------------- #
+# clocks during the timed region                                              #
+# --------------------------------------------------------------------------- #
+class ClockSampler:
+    QUERY = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+             "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+             "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        try:
+            fd, self.path = tempfile.mkstemp(suffix=".csv")
+            os.close(fd)
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.QUERY}",
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+        except (OSError, FileNotFoundError):
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        time.sleep(0.25)
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        rows = []
+        with open(self.path) as f:
+            for line in f:
+                parts = [p.strip() for p in line.split(",")]
+                if len(parts) >= 9:
+                    rows.append(parts)
+        os.unlink(self.path)
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"]}
+        sm = [float(r[1]) for r in rows if r[1].replace(".", "").isdigit()]
+        smax = [float(r[2]) for r in rows if r[2].replace(".", "").isdigit()]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in rows for i in range(4) if r[5 + i] == "Active"})
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(smax) if smax else None, "reasons": reasons,
+                "samples": len(rows)}
+
+
+# --------------------------------------------------------------------------- #
+# workload bookkeeping                                                        #
+# --------------------------------------------------------------------------- #
+def attention_bytes_per_layer(wl, seq_lens) -> int:
+    """Algorithmic HBM bytes of one verification-attention launch: every
+    visible K and V row once, Q in, O out (bf16), LSE out (fp32)."""
+    kv = int(np.sum(seq_lens.astype(np.int64))) * wl.H_kv * wl.d * 2 * 2
+    qo = wl.B * wl.rows * wl.H_q * wl.d * 2 * 2
+    return kv + qo + wl.B * wl.rows * wl.H_q * 4
+
+
+def accept_bytes(wl, mode_sampling_rows: int) -> int:
+    """Algorithmic bytes of acceptance: all (k+1) logits rows once, plus one
+    row of logits and one of q per sampled sequence for the draw."""
+    return wl.B * (wl.k + 1) * wl.V * 4 + mode_sampling_rows * wl.V * 4 * 2
+
+
+def measured_peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), "measured"
+    except (OSError, KeyError, ValueError):
+        return 6800.0, "fallback"
+
+
+# --------------------------------------------------------------------------- #
+# CPU oracle timing (the reported baseline; never the product path)           #
+# --------------------------------------------------------------------------- #
+def time_oracle_step_sample(wl, att, acc, layer: int):
+    """Oracle time of one layer of attention and of the acceptance, in s."""
+    from oracle import oracle
+    t0 = time.perf_counter()
+    oracle.verify_attention(att.q[layer], att.k_cache[layer], att.v_cache[layer],
+                            att.block_table[layer], att.seq_lens, H_kv=att.H_kv)
+    t1 = time.perf_counter()
+    oracle.accept(acc.target_logits, acc.draft_probs, acc.draft_tokens, acc.uniforms,
+                  acc.temperature)
+    t2 = time.perf_counter()
+    return t1 - t0, t2 - t1
+
+
+def oracle_cores() -> int:
+    n = os.environ.get("OMP_NUM_THREADS")
+    return int(n) if n and n.isdigit() else (os.cpu_count() or 1)
+
+
+def cpu_baseline(wl, att, acc, budget_s=12.0):
+    from oracle import oracle
+    oracle.build()
+    layers_done, t_att, t_acc, n_acc = 0, 0.0, 0.0, 0
+    start = time.perf_counter()
+    while True:
+        a, c = time_oracle_step_sample(wl, att, acc, layers_done % att.layers)
+        t_att += a
+        t_acc += c
+        layers_done += 1
+        n_acc += 1
+        if time.perf_counter() - start > budget_s or layers_done >= att.layers:
+            break
+    step_s = wl.layers * (t_att / layers_done) + t_acc / n_acc
+    return {"value": wl.B * wl.k / step_s, "unit": UNIT, "cores": oracle_cores(),
+            "kind": "oracle",
+            "sample": f"fp64 C oracle on the host: {layers_done} of {wl.layers} attention layers "
+                      f"and {n_acc} acceptance passes of the {wl.name} workload, scaled to one "
+                      f"full step ({step_s * 1e3:.1f} ms)",
+            "step_ms": step_s * 1e3}
+
+
+def run_reference(args):
+    rank, world, _ = dist_env()
+    if rank != 0:
+        return 0
+    from paper_2505_12728_gb300.workloads import (make_accept_inputs, make_attention_inputs,
+                                                  workload)
+    from oracle import oracle
+    oracle.build()
+    wl = workload(args.workload)
+    att = make_attention_inputs(wl, layers=min(wl.layers, 2))
+    acc = make_accept_inputs(wl)
+    for w in range(args.warmup):
+        time_oracle_step_sample(wl, att, acc, w % att.layers)
+    t_att, t_acc = 0.0, 0.0
+    for s in range(args.steps):
+        a, c = time_oracle_step_sample(wl, att, acc, s % att.layers)
+        t_att += a
+        t_acc += c
+    step_s = wl.layers * t_att / args.steps + t_acc / args.steps
+    value = wl.B * wl.k / step_s
+    sample = (f"each step: the fp64 C oracle on 1 of the {wl.layers} attention layers plus the "
+              f"acceptance of the {wl.name} workload; the layer time is scaled by {wl.layers}")
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT,
+            "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": step_s * 1e3, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": workload_config(wl, att.seq_lens),
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": oracle_cores(),
+                             "kind": "oracle", "sample": sample},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+def workload_config(wl, seq_lens):
+    return {"workload": wl.name, "description": wl.description, "batch": wl.B,
+            "layers": wl.layers, "H_q": wl.H_q, "H_kv": wl.H_kv, "head_dim": wl.d,
+            "draft_k": wl.k, "query_rows": wl.rows, "vocab": wl.V,
+            "prefix_tokens": [int(x) - wl.rows for x in seq_lens],
+            "page_size": 16, "acceptance": wl.mode,
+            "l2": "inputs larger than L2: every step streams "
+                  f"{wl.layers} separate KV caches"}
+
+
+# --------------------------------------------------------------------------- #
+# the GPU path                                                                #
+# --------------------------------------------------------------------------- #
+def run_ours(args):
+    import torch
+
+    rank, world, local = dist_env()
+    dist = init_dist(world, "nccl")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+
+    from paper_2505_12728_gb300 import build_lib
+    from paper_2505_12728_gb300 import specflash_verify as sfv
+    from paper_2505_12728_gb300.workloads import (make_accept_inputs, make_attention_inputs,
+                                                  workload)
+    build_lib.build()
+    sfv.load_library()
+    wl = workload(args.workload)
+    att = make_attention_inputs(wl)
+    acc = make_accept_inputs(wl)
+
+    # CPU oracle baseline first (rank 0, N = 1 only), before any GPU work
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        cpu = cpu_baseline(wl, att, acc, budget_s=args.cpu_budget)
+
+    def bf16(bits):
+        return torch.from_numpy(np.ascontiguousarray(bits).view(np.int16)).to(dev).view(
+            torch.bfloat16)
+
+    L = att.layers
+    q = bf16(att.q)                      # [L][B][n_q][H_q][d]
+    kc = [bf16(att.k_cache[l]) for l in range(L)]
+    vc = [bf16(att.v_cache[l]) for l in range(L)]
+    bt = torch.from_numpy(att.block_table).to(dev)
+    sl = torch.from_numpy(att.seq_lens).to(dev)
+    logits = torch.from_numpy(acc.target_logits).to(dev)
+    qprob = torch.from_numpy(acc.draft_probs).to(dev)
+    toks = torch.from_numpy(acc.draft_tokens).to(dev)
+    uni = torch.from_numpy(acc.uniforms).to(dev)
+    temp = torch.from_numpy(acc.temperature).to(dev)
+    out = torch.empty_like(q)
+    lse = torch.empty((L, wl.B, wl.rows, wl.H_q), dtype=torch.float32, device=dev)
+    n_acc = torch.empty(wl.B, dtype=torch.int32, device=dev)
+    out_toks = torch.empty((wl.B, wl.k + 1), dtype=torch.int32, device=dev)
+    ratio = torch.empty((wl.B, wl.k), dtype=torch.float32, device=dev)
+    ws_att = sfv.new_workspace(sfv.verify_attention_workspace_size(
+        wl.B, wl.rows, wl.H_q, wl.H_kv, wl.d, att.block_table.shape[2]), dev)
+    ws_acc = sfv.new_workspace(sfv.accept_workspace_size(wl.B, wl.k, wl.V), dev)
+    stream = torch.cuda.current_stream()
+
+    def attention_layers(qsrc):
+        for l in range(L):
+            sfv.verify_attention(qsrc[l], kc[l], vc[l], bt[l], sl, out=out[l], lse=lse[l],
+                                 workspace=ws_att, stream=stream)
+
+    def acceptance(lg, qp, tk, un, tp):
+        sfv.accept(lg, qp, tk, un, tp, num_accepted=n_acc, out_tokens=out_toks,
+                   accept_ratio=ratio, workspace=ws_acc, stream=stream)
+
+    def step():
+        attention_layers(q)
+        acceptance(logits, qprob, toks, uni, temp)
+
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+
+    # ---- device-resident timing ----
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(args.steps)]
+    clocks = ClockSampler(local)
+    clocks.start()
+    barrier(world)
+    torch.cuda.synchronize()
+    t_start = torch.cuda.Event(enable_timing=True)
+    t_end = torch.cuda.Event(enable_timing=True)
+    t_start.record(stream)
+    for s in range(args.steps):
+        ev[s][0].record(stream)
+        attention_layers(q)
+        ev[s][1].record(stream)
+        acceptance(logits, qprob, toks, uni, temp)
+        ev[s][2].record(stream)
+    t_end.record(stream)
+    torch.cuda.synchronize()
+    barrier(world)
+    clk = clocks.stop()
+    total_ms = max_over_ranks(t_start.elapsed_time(t_end), world, dev)
+    att_ms = [ev[s][0].elapsed_time(ev[s][1]) for s in range(args.steps)]
+    acc_ms = [ev[s][1].elapsed_time(ev[s][2]) for s in range(args.steps)]
+    ms_per_step = total_ms / args.steps
+    tokens = wl.B * wl.k * world * args.steps
+    value = tokens / (total_ms / 1e3)
+
+    # ---- end to end through host buffers ----
+    pin = lambda a: torch.from_numpy(np.ascontiguousarray(a)).pin_memory()
+    h_q = pin(att.q.view(np.int16))
+    h_logits, h_qprob = pin(acc.target_logits), pin(acc.draft_probs)
+    h_toks, h_uni, h_temp = pin(acc.draft_tokens), pin(acc.uniforms), pin(acc.temperature)
+    h_n = torch.empty(wl.B, dtype=torch.int32).pin_memory()
+    h_out = torch.empty((wl.B, wl.k + 1), dtype=torch.int32).pin_memory()
+    d_q = torch.empty_like(q)
+    d_logits, d_qprob = torch.empty_like(logits), torch.empty_like(qprob)
+    d_toks, d_uni, d_temp = torch.empty_like(toks), torch.empty_like(uni), torch.empty_like(temp)
+    h2d = sum(t.numel() * t.element_size() for t in (h_q, h_logits, h_qprob, h_toks, h_uni, h_temp))
+    d2h = h_n.numel() * 4 + h_out.numel() * 4
+
+    def e2e_step():
+        d_q.view(torch.int16).copy_(h_q, non_blocking=True)
+        d_logits.copy_(h_logits, non_blocking=True)
+        d_qprob.copy_(h_qprob, non_blocking=True)
+        d_toks.copy_(h_toks, non_blocking=True)
+        d_uni.copy_(h_uni, non_blocking=True)
+        d_temp.copy_(h_temp, non_blocking=True)
+        attention_layers(d_q)
+        acceptance(d_logits, d_qprob, d_toks, d_uni, d_temp)
+        h_n.copy_(n_acc, non_blocking=True)
+        h_out.copy_(out_toks, non_blocking=True)
+
+    for _ in range(args.warmup):
+        e2e_step()
+    torch.cuda.synchronize()
+    barrier(world)
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(args.steps):
+        e2e_step()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    barrier(world)
+    e2e_ms = max_over_ranks(e0.elapsed_time(e1), world, dev)
+    e2e_value = tokens / (e2e_ms / 1e3)
+
+    # ---- roofline of the dominant kernel (verification attention) ----
+    peak, peak_kind = measured_peaks()
+    bytes_layer = attention_bytes_per_layer(wl, att.seq_lens)
+    att_launch_ms = sum(att_ms) / (args.steps * L)
+    achieved = bytes_layer / (att_launch_ms / 1e3) / 1e9
+    sampling_rows = int(np.sum(acc.temperature > 0))
+    acc_launch_ms = sum(acc_ms) / args.steps
+    status = sfv.read_device_status(ws_att) | sfv.read_device_status(ws_acc)
+
+    line = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": workload_config(wl, att.seq_lens),
+        "verify_step_us": ms_per_step * 1e3,
+        "attention_us_per_layer": att_launch_ms * 1e3,
+        "accept_us": acc_launch_ms * 1e3,
+        "kv_gbs": achieved,
+        "kv_frac_of_nominal_8tbs": achieved / NOMINAL_HBM_GBS,
+        "accept_gbs": accept_bytes(wl, sampling_rows) / (acc_launch_ms / 1e3) / 1e9,
+        "mean_accepted": float(n_acc.float().mean().item()),
+        "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
+                     "frac": achieved / peak, "traffic": None,
+                     "kernel": "verify_attention_kernel",
+                     "peak_source": f"{peak_kind} copy bandwidth (MEASURED_PEAKS.json hbm_gbs)"},
+        "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d,
+                "d2h_bytes_per_step": d2h, "ms_per_step": e2e_ms / args.steps},
+        "gpu_launches": args.steps * (L + 2),
+        "clocks": clk,
+        "device_status": status,
+    }
+    if cpu is not None:
+        line["cpu_baseline"] = {k: cpu[k] for k in ("value", "unit", "cores", "kind", "sample")}
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+    return 0
+
+
+def main(argv=None):
+    ap = argparse.ArgumentParser(description=__doc__.split("\n")[0])
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--workload", default="image7b")
+    ap.add_argument("--cpu-budget", type=float, default=12.0,
+                    help="seconds of oracle work for the cpu_baseline sample")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args(argv)
+    args.warmup = max(3, args.warmup)   # at least 3 untimed warm-up steps
+    if args.impl == "reference":
+        return run_reference(args)
+    return run_ours(args)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

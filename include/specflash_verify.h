@@ -1,0 +1,165 @@
+/*
+ * specflash_verify.h -- C ABI of the GB300 (sm_103a) verification step of
+ * SpecFLASH speculative decoding (arXiv 2505.12728).
+ *
+ * The verification step has two parts (Sec. 3.1, "Preliminaries"; Sec. 3.3):
+ *   1. the target model scores the K draft tokens "in parallel within a single
+ *      forward pass": per layer, attention of the K new query rows over the
+ *      cached (mostly visual) prefix plus the causal draft block
+ *      (sf_verify_attention);
+ *   2. the token-wise acceptance-rejection rule: candidate T'_i is kept with
+ *      probability min(1, p_i/q_i), candidates after the first rejection are
+ *      discarded, and the token at the rejected position is drawn from the
+ *      residual distribution norm(max(0, p - q)); at temperature 0 (greedy
+ *      decoding, Sec. 4.2) a candidate is kept iff it is the target argmax
+ *      (sf_accept).
+ *
+ * Conventions for every entry point:
+ *   - Pointers are DEVICE pointers unless stated otherwise.  The caller owns
+ *     every buffer; the library never allocates, frees or synchronises, and
+ *     enqueues its kernels on `stream` (0 = the legacy default stream).
+ *   - Return value: SF_OK (0) or an sf_status code.  Argument errors are
+ *     detected on the host before any launch; nothing is enqueued then.
+ *     sf_last_error() gives a thread-local description of the last failure.
+ *   - Data errors that only the device can see (a page index outside the
+ *     pool, a draft token outside [0, V)) never fault: the offending access
+ *     is replaced by a zero page / a rejection, and a bit is set in the
+ *     status word at the start of the workspace (SF_DEVICE_* below), which
+ *     sf_read_device_status() returns.
+ *   - Workspaces must be zero-filled once before their first use
+ *     (sf_workspace_init, or cudaMemset to 0).  The kernels leave their
+ *     counters at zero on exit, so a workspace can be reused by later calls
+ *     on the same stream; calls that overlap on the GPU must use distinct
+ *     workspaces.  Re-initialise after a nonzero device status.
+ *   - Results are deterministic: for fixed shapes, inputs and num_splits they
+ *     are bit-identical from run to run (no floating-point atomics).
+ */
+#ifndef SPECFLASH_VERIFY_H
+#define SPECFLASH_VERIFY_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#include <cuda_runtime_api.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  SF_OK = 0,
+  SF_ERR_INVALID_ARG = 1,   /* bad shape, NULL pointer, misaligned buffer      */
+  SF_ERR_UNSUPPORTED = 2,   /* valid but not built: head_dim, page size, ...   */
+  SF_ERR_CUDA = 3,          /* a CUDA runtime/driver call failed               */
+  SF_ERR_WORKSPACE = 4,     /* workspace NULL or smaller than required         */
+  SF_ERR_DEVICE_STATUS = 5  /* the device status word is nonzero               */
+} sf_status;
+
+/* Bits of the device status word (first 4 bytes of every workspace). */
+#define SF_DEVICE_BAD_PAGE 0x1u  /* block_table entry outside [0, num_pages)  */
+#define SF_DEVICE_BAD_TOKEN 0x2u /* draft token outside [0, V)                */
+#define SF_DEVICE_TIMEOUT 0x4u   /* a bounded wait on a copy gave up (~1 s)   */
+#define SF_DEVICE_BAD_SEQLEN 0x8u /* seq_lens[b] outside [n_q, max_pages*16]   */
+
+/* Limits of this build. */
+#define SF_PAGE_SIZE 16      /* tokens per KV page                            */
+#define SF_MAX_BATCH 1024    /* sequences per call                            */
+#define SF_MAX_QUERY_ROWS 16 /* n_q: draft rows scored per sequence           */
+#define SF_MAX_GROUP 8       /* H_q / H_kv                                    */
+#define SF_MAX_DRAFT 16      /* k: draft length                               */
+
+/* Static string naming a status code. */
+const char *sf_status_string(int status);
+
+/* Thread-local, human-readable detail of the last failing call ("" if none). */
+const char *sf_last_error(void);
+
+/* Library version: major * 10000 + minor * 100 + patch. */
+int sf_version(void);
+
+/* Zero-fill `bytes` of `workspace` on `stream` (asynchronous). */
+int sf_workspace_init(void *workspace, size_t bytes, cudaStream_t stream);
+
+/* Synchronously read the device status word of a workspace (tests and
+ * diagnostics only: it waits for all work on the device).  On success
+ * *status_out holds the SF_DEVICE_* bits; returns SF_OK or SF_ERR_CUDA. */
+int sf_read_device_status(const void *workspace, uint32_t *status_out);
+
+/* ------------------------------------------------------------------------ */
+/* Verification attention (Sec. 3.1: "computes the probabilities of these K  */
+/* candidate tokens in parallel within a single forward pass"; the verify    */
+/* costs about one target step, Eq. 1).                                      */
+/*                                                                           */
+/* For each sequence b, draft row i < n_q and query head h (KV head          */
+/* h / (H_q / H_kv)): the visible keys are the L_b = seq_lens[b] - n_q       */
+/* cached prefix tokens (visual first, then text) plus draft rows 0..i,      */
+/* s_t = softmax_scale * <q, k_t>, lse = ln sum_t exp(s_t),                  */
+/* out = sum_t exp(s_t - lse) * v_t.                                         */
+/*                                                                           */
+/* q            bf16 [B][n_q][H_q][head_dim], already position-encoded.      */
+/* k_cache      bf16 [num_pages][H_kv][page_size][head_dim]; 16-byte aligned */
+/* v_cache      bf16, same layout as k_cache.                                */
+/* block_table  int32 [B][max_pages_per_seq]: logical page -> physical page. */
+/*              Entries past a sequence's last page are never read.          */
+/* seq_lens     int32 [B]: L_b + n_q, the draft rows' K/V already written at */
+/*              positions L_b..L_b+n_q-1.  Must satisfy                      */
+/*              n_q <= seq_lens[b] <= max_pages_per_seq * page_size; values  */
+/*              outside are clamped and flagged with SF_DEVICE_BAD_SEQLEN.   */
+/* head_dim     64 or 128; page_size 16; 1 <= n_q <= 16; H_q % H_kv == 0,    */
+/*              H_q / H_kv <= 8; 1 <= B <= 1024.                             */
+/* softmax_scale  0 selects 1/sqrt(head_dim).                                */
+/* num_splits   number of cooperating CTAs the batch's KV tiles are divided */
+/*              among; 0 picks (SM count x resident CTAs per SM).  The        */
+/*              result depends on it only through rounding.                 */
+/* out          bf16 [B][n_q][H_q][head_dim].                                */
+/* lse          fp32 [B][n_q][H_q] (natural log, scaled scores); may be NULL.*/
+/* workspace    >= sf_verify_attention_workspace_size(...) bytes, 256-byte   */
+/*              aligned, zero-filled before first use.                       */
+/* ------------------------------------------------------------------------ */
+size_t sf_verify_attention_workspace_size(int B, int n_q, int H_q, int H_kv, int head_dim,
+                                          int max_pages_per_seq, int page_size,
+                                          int num_splits);
+
+int sf_verify_attention(const void *q, const void *k_cache, const void *v_cache,
+                        const int32_t *block_table, const int32_t *seq_lens, int B, int n_q,
+                        int H_q, int H_kv, int head_dim, int page_size, int num_pages,
+                        int max_pages_per_seq, float softmax_scale, int num_splits, void *out,
+                        float *lse, void *workspace, size_t workspace_bytes,
+                        cudaStream_t stream);
+
+/* ------------------------------------------------------------------------ */
+/* Acceptance (Sec. 3.1: acceptance probability as the ratio of target to    */
+/* draft probability, discard from the first rejection on, resample from the */
+/* residual distribution; Sec. 3.3: "the standard token-wise acceptance-     */
+/* rejection rule"; Sec. 4.2: tau = 0 is greedy decoding).                   */
+/*                                                                           */
+/* target_logits fp32 [B][k+1][V]: row i < k scores draft T'_{i+1}; row k is */
+/*               the bonus row used when all k drafts are accepted.          */
+/* draft_probs   fp32 [B][k][V]: draft distributions q_i, used as given.     */
+/* draft_tokens  int32 [B][k].                                               */
+/* uniforms      fp32 [B][k+1] in [0,1): u_i for test i, u_k for the draw.   */
+/* temperature   fp32 [B]: p = softmax(logits / tau); tau <= 0 selects       */
+/*               greedy matching for that sequence (mixed batches allowed).  */
+/* num_accepted  int32 [B] in [0, k].                                        */
+/* out_tokens    int32 [B][k+1]: the accepted drafts, then the corrected     */
+/*               (or bonus) token; entries past num_accepted are -1.         */
+/* accept_ratio  fp32 [B][k] = min(1, p_i(T'_i)/q_i(T'_i)) for every i      */
+/*               (greedy: 1 on a match, else 0); may be NULL.                */
+/* Rule details: accept iff u_i * q < p (strict); greedy ties go to the      */
+/* lowest token id; a residual with zero mass falls back to p_j; the draw is */
+/* the smallest token x with u_k * S < C(x) in ascending token order.        */
+/* Limits: 1 <= B <= 1024, 1 <= k <= 16, 2 <= V < 2^31 / (k + 1).            */
+/* ------------------------------------------------------------------------ */
+size_t sf_accept_workspace_size(int B, int k, int V);
+
+int sf_accept(const float *target_logits, const float *draft_probs,
+              const int32_t *draft_tokens, const float *uniforms, const float *temperature,
+              int B, int k, int V, int32_t *num_accepted, int32_t *out_tokens,
+              float *accept_ratio, void *workspace, size_t workspace_bytes,
+              cudaStream_t stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* SPECFLASH_VERIFY_H */

@@ -1,0 +1,39 @@
+// sf_host.h -- host-side helpers shared by the C-ABI translation units:
+// thread-local error text, per-device properties, TMA descriptor encoding.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <stddef.h>
+#include <stdint.h>
+
+#include "specflash_verify.h"
+
+namespace sf {
+
+// Records a formatted message as the calling thread's last error and returns
+// `status` (so call sites can `return fail(SF_ERR_..., "...")`).
+int fail(int status, const char *fmt, ...);
+void clear_error();
+
+// Properties of the current device, cached per device ordinal.
+struct DeviceInfo {
+  int ordinal = -1;
+  int sm_count = 0;
+  int max_smem_optin = 0;
+  int cc_major = 0, cc_minor = 0;
+};
+int current_device(DeviceInfo *info);
+
+// cuTensorMapEncodeTiled fetched through the runtime (no link-time libcuda).
+int encode_tensor_map_2d_bf16(CUtensorMap *map, const void *base, uint64_t inner_elems,
+                              uint64_t rows, uint64_t row_stride_bytes, uint32_t box_inner,
+                              uint32_t box_rows, bool swizzle_128b);
+
+inline bool aligned(const void *p, size_t a) {
+  return (reinterpret_cast<uintptr_t>(p) % a) == 0;
+}
+
+inline size_t round_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+}  // namespace sf

@@ -1,0 +1,768 @@
+// verify_attention.cu -- split-KV verification attention for sm_103a.
+//
+// The target model scores the K draft tokens in one forward pass against its
+// cache of visual-then-text tokens (Sec. 3.1; verification costs about one
+// target step, Eq. 1).  Per layer that is attention of n_q new query rows per
+// sequence over the prefix plus the causal draft block:
+//   out[b,i,h] = sum_t softmax_t(scale * <q[b,i,h], k[b,t,h/g]>) v[b,t,h/g],
+//   t = 0 .. L_b + i,   L_b = seq_lens[b] - n_q.
+//
+// GB300 design (the paper gives no kernel; its runs used one A6000):
+//  * Work unit = a tile of 64 cached tokens of one (sequence, KV head)
+//    "segment".  All tiles of the batch form one ordered list that is cut
+//    into G equal, contiguous ranges, one per CTA (G = SMs x resident CTAs),
+//    so long and short sequences balance without any host-side knowledge of
+//    seq_lens.  A CTA's range touches one or two segments ("pieces").
+//  * Each CTA streams its tiles through a STAGES-deep ring in shared memory:
+//    one elected warp issues 2-D TMA copies of whole 16-token pages (128-byte
+//    swizzled boxes, one per page, half head_dim and tensor) straight from
+//    the block table into the ring, completing on an mbarrier; nothing else
+//    touches HBM in the loop.
+//  * All n_q * g query rows of a KV head share each K/V tile.  The rows are
+//    the M dimension of bf16 m16n8k16 tensor-core MMAs (S = Q K^T and
+//    O += P V, fp32 accumulate); scores stay in registers, where an fp32
+//    online softmax (base-2, scale folded in) rescales the running output.
+//    With one row tile (MHA, n_q <= 16) the four warps split the tile's keys
+//    and combine in shared memory at the end of a piece.
+//  * A piece that covers a whole segment writes bf16 out and fp32 LSE
+//    directly.  Otherwise it writes an fp32 partial (O unnormalised, running
+//    max, running sum) to the workspace, and the CTA that takes the last
+//    ticket of the segment (an atomic counter; nobody waits) merges all
+//    partials in piece order, so results are deterministic.
+//  * Page indices outside the pool and positions past a sequence's end are
+//    loaded as zero boxes (TMA out-of-bounds fill); bad indices set a bit in
+//    the status word.  Every mbarrier wait is bounded.
+#include <cmath>
+#include <mutex>
+
+#include "sf_device.cuh"
+#include "sf_host.h"
+
+namespace sf {
+
+constexpr int kTileTokens = 64;            // keys per ring stage
+constexpr int kPageTokens = SF_PAGE_SIZE;  // 16
+constexpr int kPagesPerTile = kTileTokens / kPageTokens;
+constexpr int kRowBytes = 128;             // one swizzled smem row (64 bf16)
+constexpr int kHalfBytes = kTileTokens * kRowBytes;  // 64 tokens x 128 B
+constexpr int kBeyondEnd = -2147483647 - 1;           // page past the sequence end
+
+struct AttnParams {
+  const __nv_bfloat16 *q;
+  const int32_t *block_table;
+  const int32_t *seq_lens;
+  __nv_bfloat16 *out;
+  float *lse;
+  uint32_t *status;
+  uint32_t *tickets;  // [B * H_kv]
+  float *partials;    // [G + B * H_kv][R][D + 2]
+  int B, n_q, H_q, H_kv, group, R;
+  int num_pages, max_pages, max_tokens;
+  int oob_row;        // a tensor-map row beyond the pool: loads as zeros
+  float scale_log2;   // softmax_scale * log2(e)
+  int G;
+  int slot_stride;    // floats per partial slot: R*D (O) + R (max) + R (sum), padded to 4
+};
+
+// Floats per partial slot; a multiple of 4 so every slot starts 16-byte aligned.
+__host__ __device__ inline int partial_slot_floats(int R, int D) {
+  return (R * (D + 2) + 3) / 4 * 4;
+}
+
+// Byte offset of 16-byte chunk `c` (head_dim / 8 index) of token `t` inside a
+// tile written by 128B-swizzled TMA boxes: [c / 8][t][(c % 8) ^ (t % 8)].
+__device__ __forceinline__ uint32_t swz(int t, int c) {
+  return static_cast<uint32_t>((c >> 3) * kHalfBytes + t * kRowBytes +
+                               (((c & 7) ^ (t & 7)) << 4));
+}
+
+template <int D, int STAGES, int NW>
+struct AttnSmem {
+  static constexpr int kTensorTileBytes = kTileTokens * D * 2;
+  static constexpr int kStageBytes = 2 * kTensorTileBytes;
+  static constexpr int kRingBytes = STAGES * kStageBytes;
+  // ring | STAGES mbarriers | misc ints | tiles prefix [B+1] | seq lens [B]
+  static constexpr int kBarOffset = kRingBytes;
+  static constexpr int kMiscOffset = kBarOffset + 8 * STAGES;
+  static constexpr int kMiscInts = 8 + 2 * NW;
+  static constexpr int kPrefixOffset = kMiscOffset + 4 * kMiscInts;
+  static int bytes(int B) { return 1024 + kPrefixOffset + 4 * (2 * B + 2); }
+};
+
+// Exclusive prefix of per-sequence tile counts into s_prefix[0..B], clamped
+// sequence lengths into s_len[0..B-1].
+template <int NT>
+__device__ void tile_prefix(const AttnParams &p, int *s_prefix, int *s_len, int *s_warp) {
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int per = (p.B + NT - 1) / NT;
+  const int b0 = tid * per;
+  int local = 0;
+  for (int b = b0; b < b0 + per && b < p.B; ++b) {
+    int T = p.seq_lens[b];
+    if (T < p.n_q || T > p.max_tokens) {
+      set_status(p.status, SF_DEVICE_BAD_SEQLEN);
+      T = T < p.n_q ? p.n_q : p.max_tokens;
+    }
+    s_len[b] = T;
+    local += (T + kTileTokens - 1) / kTileTokens;
+  }
+  int incl = local;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    int v = __shfl_up_sync(0xffffffffu, incl, o);
+    if (lane >= o) incl += v;
+  }
+  if (lane == 31) s_warp[warp] = incl;
+  __syncthreads();
+  int warp_off = 0;
+  for (int w = 0; w < warp; ++w) warp_off += s_warp[w];
+  int run = warp_off + incl - local;
+  for (int b = b0; b < b0 + per && b < p.B; ++b) {
+    s_prefix[b] = run;
+    run += (s_len[b] + kTileTokens - 1) / kTileTokens;
+  }
+  if (tid == NT - 1) s_prefix[p.B] = warp_off + incl;
+}
+
+// Sequence b owning global tile t: H_kv * s_prefix[b] <= t < H_kv * s_prefix[b+1].
+__device__ __forceinline__ int find_sequence(long long t, const int *s_prefix, int B, int H_kv) {
+  int lo = 0, hi = B - 1;
+  while (lo < hi) {
+    int mid = (lo + hi + 1) >> 1;
+    if ((long long)H_kv * s_prefix[mid] <= t) lo = mid; else hi = mid - 1;
+  }
+  return lo;
+}
+
+// CTA whose range [c*Tot/G, (c+1)*Tot/G) contains global tile t.
+__device__ __forceinline__ int owner_cta(long long t, long long Tot, int G) {
+  return static_cast<int>(((t + 1) * G - 1) / Tot);
+}
+
+template <int D, int KS, int NW, int STAGES>
+__global__ void __launch_bounds__(NW * 32, (NW == 4 ? 2 : 1))
+verify_attention_kernel(const __grid_constant__ CUtensorMap tmap_k,
+                        const __grid_constant__ CUtensorMap tmap_v,
+                        const __grid_constant__ AttnParams p) {
+  using L = AttnSmem<D, STAGES, NW>;
+  constexpr int NTHREADS = NW * 32;
+  constexpr int RT_SLOTS = NW / KS;      // row tiles a CTA covers at once
+  constexpr int KW = kTileTokens / KS;   // keys per warp per tile
+  constexpr int NT = KW / 8;             // score n-tiles per warp
+  constexpr int KK = D / 16;             // k-steps of Q K^T
+  constexpr int DT = D / 8;              // output n-tiles
+  constexpr int HALVES = D / 64;
+  constexpr float kLn2 = 0.6931471805599453f;
+
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t *smem = reinterpret_cast<uint8_t *>(
+      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+  const uint32_t ring = smem_addr(smem);
+  const uint32_t bar0 = ring + L::kBarOffset;
+  int *s_misc = reinterpret_cast<int *>(smem + L::kMiscOffset);
+  int *s_prefix = reinterpret_cast<int *>(smem + L::kPrefixOffset);
+  int *s_len = s_prefix + p.B + 1;
+
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int rt = warp % RT_SLOTS, ks = warp / RT_SLOTS;
+  const int row_tiles = (p.R + 15) >> 4;
+  const bool active = rt < row_tiles;
+
+  if (tid == 0) {
+    for (int s = 0; s < STAGES; ++s) mbar_init(bar0 + 8 * s, 1);
+    fence_mbar_init();
+    prefetch_tensormap(&tmap_k);
+    prefetch_tensormap(&tmap_v);
+  }
+  tile_prefix<NTHREADS>(p, s_prefix, s_len, s_misc + 8);
+  __syncthreads();
+
+  // The host sizes the grid from an upper bound of the tile count; with more
+  // CTAs than tiles the surplus CTAs leave, so that every CTA of the
+  // partition owns at least one tile and a segment's pieces are owned by
+  // consecutive CTAs.
+  const long long Tot = (long long)p.H_kv * s_prefix[p.B];
+  const int G = Tot < (long long)p.G ? static_cast<int>(Tot) : p.G;
+  if (static_cast<int>(blockIdx.x) >= G) return;
+  const long long t_begin = (long long)blockIdx.x * Tot / G;
+  const long long t_end = (long long)(blockIdx.x + 1) * Tot / G;
+
+  const uint64_t policy = l2_policy_evict_first();
+  uint32_t consumed = 0;  // tiles consumed by this CTA so far (ring position)
+  bool timed_out = false;
+
+  for (long long t = t_begin; t < t_end && !timed_out;) {
+    // ---- locate the piece: segment (b, h_kv), local tiles [lt0, lt1) ----
+    const int b = find_sequence(t, s_prefix, p.B, p.H_kv);
+    const int tiles_b = s_prefix[b + 1] - s_prefix[b];
+    const long long seg_base = (long long)p.H_kv * s_prefix[b];
+    const int h_kv = static_cast<int>((t - seg_base) / tiles_b);
+    const int lt0 = static_cast<int>((t - seg_base) % tiles_b);
+    const long long left = t_end - t;
+    const int n_tiles = left < (long long)(tiles_b - lt0) ? static_cast<int>(left) : tiles_b - lt0;
+    const long long seg_first = seg_base + (long long)h_kv * tiles_b;
+    const int seg = b * p.H_kv + h_kv;
+    const int c_first = owner_cta(seg_first, Tot, G);
+    const int c_last = owner_cta(seg_first + tiles_b - 1, Tot, G);
+    const int n_pieces = c_last - c_first + 1;
+    const int T = s_len[b];
+    const int Lb = T - p.n_q;
+    t += n_tiles;
+
+    // ---- producer: lanes 0..3 of warp 0 own the four pages of a tile ----
+    // fetch_page reads the block table (the value is checked only when the
+    // copy is issued, so the load latency overlaps the current tile's math)
+    auto fetch_page = [&](int lt, int pg) -> int {
+      const int lp = lt * kPagesPerTile + pg;
+      if (lp * kPageTokens >= T) return kBeyondEnd;
+      return p.block_table[(size_t)b * p.max_pages + lp];
+    };
+    auto issue = [&](int slot, int pg, int phys) {
+      // one page (16 tokens) of K and V into ring slot `slot`; pages past the
+      // end of the sequence or outside the pool load as zeros
+      int row = p.oob_row;
+      if (phys != kBeyondEnd) {
+        if (phys < 0 || phys >= p.num_pages) set_status(p.status, SF_DEVICE_BAD_PAGE);
+        else row = (phys * p.H_kv + h_kv) * kPageTokens;
+      }
+      const uint32_t dst = ring + slot * L::kStageBytes + pg * kPageTokens * kRowBytes;
+      const uint32_t bar = bar0 + 8 * slot;
+#pragma unroll
+      for (int hf = 0; hf < HALVES; ++hf) {
+        tma_load_2d(dst + hf * kHalfBytes, &tmap_k, hf * 64, row, bar, policy);
+        tma_load_2d(dst + L::kTensorTileBytes + hf * kHalfBytes, &tmap_v, hf * 64, row, bar,
+                    policy);
+      }
+    };
+
+    const int prologue = n_tiles < STAGES ? n_tiles : STAGES;
+    const uint32_t piece_base = consumed;  // ring position of the piece's first tile
+    int issued = prologue;                 // tiles of this piece issued so far
+    int next_phys = 0;  // lanes 0..3 of warp 0: block-table entry of the next tile
+    if (warp == 0) {
+      if (lane < prologue) mbar_arrive_expect_tx(bar0 + 8 * ((piece_base + lane) % STAGES),
+                                                 L::kStageBytes);
+      __syncwarp();
+      if (lane < kPagesPerTile * prologue) {
+        const int j = lane / kPagesPerTile, pg = lane % kPagesPerTile;
+        issue((piece_base + j) % STAGES, pg, fetch_page(lt0 + j, pg));
+      }
+      if (lane < kPagesPerTile && prologue < n_tiles) next_phys = fetch_page(lt0 + prologue, lane);
+    }
+
+    // ---- consumers: Q fragments of this warp's 16 rows ----
+    // row r = i * g + j  <->  (draft row i, query head h_kv * g + j)
+    const int r0 = rt * 16 + (lane >> 2), r1 = r0 + 8;
+    uint32_t qa[KK][4];
+    {
+      const int cols = 2 * (lane & 3);
+      auto qptr = [&](int r) -> const __nv_bfloat16 * {
+        const int i = r / p.group, j = r % p.group;
+        return p.q + (((size_t)b * p.n_q + i) * p.H_q + (size_t)h_kv * p.group + j) * D;
+      };
+      const bool v0 = active && r0 < p.R, v1 = active && r1 < p.R;
+      const __nv_bfloat16 *q0 = v0 ? qptr(r0) : nullptr;
+      const __nv_bfloat16 *q1 = v1 ? qptr(r1) : nullptr;
+#pragma unroll
+      for (int kk = 0; kk < KK; ++kk) {
+        const int c = kk * 16 + cols;
+        qa[kk][0] = v0 ? *reinterpret_cast<const uint32_t *>(q0 + c) : 0u;
+        qa[kk][1] = v1 ? *reinterpret_cast<const uint32_t *>(q1 + c) : 0u;
+        qa[kk][2] = v0 ? *reinterpret_cast<const uint32_t *>(q0 + c + 8) : 0u;
+        qa[kk][3] = v1 ? *reinterpret_cast<const uint32_t *>(q1 + c + 8) : 0u;
+      }
+    }
+    // last visible key position of each of the thread's two rows
+    const int lim0 = Lb + min(r0 / p.group, p.n_q - 1);
+    const int lim1 = Lb + min(r1 / p.group, p.n_q - 1);
+
+    float m0 = -INFINITY, m1 = -INFINITY, l0 = 0.f, l1 = 0.f;
+    float o[DT][4];
+#pragma unroll
+    for (int dt = 0; dt < DT; ++dt) o[dt][0] = o[dt][1] = o[dt][2] = o[dt][3] = 0.f;
+
+    for (int it = 0; it < n_tiles; ++it) {
+      const int slot = consumed % STAGES;
+      const uint32_t parity = (consumed / STAGES) & 1u;
+      const int lt = lt0 + it;
+      const bool ok = mbar_wait_bounded(bar0 + 8 * slot, parity);
+      const uint32_t kbase = ring + slot * L::kStageBytes;
+      const uint32_t vbase = kbase + L::kTensorTileBytes;
+      const int tile_pos = lt * kTileTokens;
+
+      // Positions past the sequence end inside its last page hold whatever
+      // the cache page holds; zero those V rows so that 0 * v stays 0.
+      const int valid = T - tile_pos;
+      if (valid < kTileTokens) {
+        if (ok) {
+          uint8_t *vt = smem + slot * L::kStageBytes + L::kTensorTileBytes;
+          for (int idx = tid; idx < (kTileTokens - valid) * HALVES * 8; idx += NTHREADS) {
+            const int tok = valid + idx / (HALVES * 8);
+            const int rem = idx % (HALVES * 8);
+            *reinterpret_cast<uint4 *>(vt + (rem >> 3) * kHalfBytes + tok * kRowBytes +
+                                       (rem & 7) * 16) = make_uint4(0, 0, 0, 0);
+          }
+          fence_proxy_async_smem();
+        }
+        asm volatile("bar.sync 1, %0;" ::"n"(NTHREADS) : "memory");
+      }
+
+      if (ok && active) {
+        float s[NT][4];
+#pragma unroll
+        for (int nt = 0; nt < NT; ++nt) s[nt][0] = s[nt][1] = s[nt][2] = s[nt][3] = 0.f;
+        // S = Q K^T over this warp's KW keys
+#pragma unroll
+        for (int kk = 0; kk < KK; kk += 2) {
+#pragma unroll
+          for (int nt = 0; nt < NT; ++nt) {
+            const int key = ks * KW + nt * 8 + (lane & 7);
+            uint32_t b0, b1, b2, b3;
+            ldmatrix_x4(kbase + swz(key, 2 * kk + (lane >> 3)), b0, b1, b2, b3);
+            mma_bf16_16816(s[nt], qa[kk], b0, b1);
+            mma_bf16_16816(s[nt], qa[kk + 1], b2, b3);
+          }
+        }
+        // causal mask of the draft block (and of positions past the end)
+        if (tile_pos + kTileTokens - 1 > Lb) {
+#pragma unroll
+          for (int nt = 0; nt < NT; ++nt) {
+            const int kp = tile_pos + ks * KW + nt * 8 + 2 * (lane & 3);
+            if (kp > lim0) s[nt][0] = -INFINITY;
+            if (kp + 1 > lim0) s[nt][1] = -INFINITY;
+            if (kp > lim1) s[nt][2] = -INFINITY;
+            if (kp + 1 > lim1) s[nt][3] = -INFINITY;
+          }
+        }
+        // online softmax in base 2 with the scale folded in
+        float mx0 = -INFINITY, mx1 = -INFINITY;
+#pragma unroll
+        for (int nt = 0; nt < NT; ++nt) {
+          mx0 = fmaxf(mx0, fmaxf(s[nt][0], s[nt][1]));
+          mx1 = fmaxf(mx1, fmaxf(s[nt][2], s[nt][3]));
+        }
+        mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, 1));
+        mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, 2));
+        mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 1));
+        mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 2));
+        const float mn0 = fmaxf(m0, mx0 * p.scale_log2);
+        const float mn1 = fmaxf(m1, mx1 * p.scale_log2);
+        const float mu0 = mn0 == -INFINITY ? 0.f : mn0;
+        const float mu1 = mn1 == -INFINITY ? 0.f : mn1;
+        const float a0 = exp2f(m0 - mu0), a1 = exp2f(m1 - mu1);
+        m0 = mn0;
+        m1 = mn1;
+        float rs0 = 0.f, rs1 = 0.f;
+#pragma unroll
+        for (int nt = 0; nt < NT; ++nt) {
+          s[nt][0] = exp2f(fmaf(s[nt][0], p.scale_log2, -mu0));
+          s[nt][1] = exp2f(fmaf(s[nt][1], p.scale_log2, -mu0));
+          s[nt][2] = exp2f(fmaf(s[nt][2], p.scale_log2, -mu1));
+          s[nt][3] = exp2f(fmaf(s[nt][3], p.scale_log2, -mu1));
+          rs0 += s[nt][0] + s[nt][1];
+          rs1 += s[nt][2] + s[nt][3];
+        }
+        l0 = l0 * a0 + rs0;
+        l1 = l1 * a1 + rs1;
+#pragma unroll
+        for (int dt = 0; dt < DT; ++dt) {
+          o[dt][0] *= a0;
+          o[dt][1] *= a0;
+          o[dt][2] *= a1;
+          o[dt][3] *= a1;
+        }
+        // O += P V
+#pragma unroll
+        for (int kt = 0; kt < KW / 16; ++kt) {
+          uint32_t pa[4];
+          pa[0] = pack_bf16x2(s[2 * kt][0], s[2 * kt][1]);
+          pa[1] = pack_bf16x2(s[2 * kt][2], s[2 * kt][3]);
+          pa[2] = pack_bf16x2(s[2 * kt + 1][0], s[2 * kt + 1][1]);
+          pa[3] = pack_bf16x2(s[2 * kt + 1][2], s[2 * kt + 1][3]);
+          const int key = ks * KW + kt * 16 + (lane & 7) + ((lane >> 3) & 1) * 8;
+#pragma unroll
+          for (int dt = 0; dt < DT; dt += 2) {
+            uint32_t b0, b1, b2, b3;
+            ldmatrix_x4_trans(vbase + swz(key, dt + (lane >> 4)), b0, b1, b2, b3);
+            mma_bf16_16816(o[dt], pa, b0, b1);
+            mma_bf16_16816(o[dt + 1], pa, b2, b3);
+          }
+        }
+      }
+      // every warp is done with this slot; refill it with tile it + STAGES
+      timed_out = __syncthreads_or(!ok) != 0;
+      ++consumed;
+      if (timed_out) break;
+      if (it + STAGES < n_tiles) {
+        if (warp == 0) {
+          const int nslot = (consumed - 1) % STAGES;
+          if (lane == 0) mbar_arrive_expect_tx(bar0 + 8 * nslot, L::kStageBytes);
+          __syncwarp();
+          if (lane < kPagesPerTile) {
+            issue(nslot, lane, next_phys);
+            if (it + STAGES + 1 < n_tiles) next_phys = fetch_page(lt0 + it + STAGES + 1, lane);
+          }
+        }
+        ++issued;
+      }
+    }
+    if (timed_out) {
+      // Unwind: wait (bounded) for the copies still in flight -- the tile
+      // that timed out and any issued after it -- then leave.
+      if (tid == 0) {
+        set_status(p.status, SF_DEVICE_TIMEOUT);
+        for (uint32_t x = consumed - 1; x < piece_base + (uint32_t)issued; ++x)
+          (void)mbar_wait_bounded(bar0 + 8 * (x % STAGES), (x / STAGES) & 1u);
+      }
+      __syncthreads();
+      return;
+    }
+
+    // ---- finish the piece ----
+    l0 += __shfl_xor_sync(0xffffffffu, l0, 1);
+    l0 += __shfl_xor_sync(0xffffffffu, l0, 2);
+    l1 += __shfl_xor_sync(0xffffffffu, l1, 1);
+    l1 += __shfl_xor_sync(0xffffffffu, l1, 2);
+
+    if constexpr (KS > 1) {
+      // warps ks >= 1 hand their (m, l, O) to warp ks == 0 of the same row
+      // tile through the (now idle) ring memory
+      constexpr int kPer = 4 * DT + 4;
+      float *xchg = reinterpret_cast<float *>(smem);
+      if (active && ks > 0) {
+        float *dst = xchg + ((size_t)(rt * (KS - 1) + ks - 1) * 32 + lane) * kPer;
+#pragma unroll
+        for (int dt = 0; dt < DT; ++dt)
+          *reinterpret_cast<float4 *>(dst + 4 * dt) = make_float4(o[dt][0], o[dt][1], o[dt][2], o[dt][3]);
+        *reinterpret_cast<float4 *>(dst + 4 * DT) = make_float4(m0, m1, l0, l1);
+      }
+      __syncthreads();
+      if (active && ks == 0) {
+        float M0 = m0, M1 = m1;
+        for (int s2 = 1; s2 < KS; ++s2) {
+          const float4 ml = *reinterpret_cast<const float4 *>(
+              xchg + ((size_t)(rt * (KS - 1) + s2 - 1) * 32 + lane) * kPer + 4 * DT);
+          M0 = fmaxf(M0, ml.x);
+          M1 = fmaxf(M1, ml.y);
+        }
+        // a row may see no key at all in this piece (every key masked):
+        // then every max is -inf and the reference must be finite
+        const float U0 = M0 == -INFINITY ? 0.f : M0, U1 = M1 == -INFINITY ? 0.f : M1;
+        const float w0 = exp2f(m0 - U0), w1 = exp2f(m1 - U1);
+        l0 *= w0;
+        l1 *= w1;
+#pragma unroll
+        for (int dt = 0; dt < DT; ++dt) {
+          o[dt][0] *= w0; o[dt][1] *= w0; o[dt][2] *= w1; o[dt][3] *= w1;
+        }
+        for (int s2 = 1; s2 < KS; ++s2) {
+          const float *src = xchg + ((size_t)(rt * (KS - 1) + s2 - 1) * 32 + lane) * kPer;
+          const float4 ml = *reinterpret_cast<const float4 *>(src + 4 * DT);
+          const float v0 = exp2f(ml.x - U0), v1 = exp2f(ml.y - U1);
+          l0 += ml.z * v0;
+          l1 += ml.w * v1;
+#pragma unroll
+          for (int dt = 0; dt < DT; ++dt) {
+            const float4 x = *reinterpret_cast<const float4 *>(src + 4 * dt);
+            o[dt][0] += x.x * v0; o[dt][1] += x.y * v0; o[dt][2] += x.z * v1; o[dt][3] += x.w * v1;
+          }
+        }
+        m0 = M0;
+        m1 = M1;
+      }
+      fence_proxy_async_smem();  // generic writes to the ring before later TMA writes
+      __syncthreads();           // the ring is refilled by the next piece's prologue
+    }
+
+    const bool writer = active && ks == 0;
+    const int colb = 2 * (lane & 3);
+    if (n_pieces == 1) {
+      // the whole segment is in this CTA: normalise and write
+      if (writer) {
+        const float inv0 = 1.f / l0, inv1 = 1.f / l1;
+        auto orow = [&](int r) -> __nv_bfloat16 * {
+          const int i = r / p.group, j = r % p.group;
+          return p.out + (((size_t)b * p.n_q + i) * p.H_q + (size_t)h_kv * p.group + j) * D;
+        };
+        if (r0 < p.R) {
+          __nv_bfloat16 *dst = orow(r0);
+#pragma unroll
+          for (int dt = 0; dt < DT; ++dt)
+            *reinterpret_cast<uint32_t *>(dst + dt * 8 + colb) = pack_bf16x2(o[dt][0] * inv0, o[dt][1] * inv0);
+        }
+        if (r1 < p.R) {
+          __nv_bfloat16 *dst = orow(r1);
+#pragma unroll
+          for (int dt = 0; dt < DT; ++dt)
+            *reinterpret_cast<uint32_t *>(dst + dt * 8 + colb) = pack_bf16x2(o[dt][2] * inv1, o[dt][3] * inv1);
+        }
+        if (p.lse && (lane & 3) == 0) {
+          auto lidx = [&](int r) {
+            const int i = r / p.group, j = r % p.group;
+            return ((size_t)b * p.n_q + i) * p.H_q + (size_t)h_kv * p.group + j;
+          };
+          if (r0 < p.R) p.lse[lidx(r0)] = (m0 + log2f(l0)) * kLn2;
+          if (r1 < p.R) p.lse[lidx(r1)] = (m1 + log2f(l1)) * kLn2;
+        }
+      }
+      continue;
+    }
+
+    // ---- several pieces: write this piece's partial, take a ticket ----
+    const int piece = static_cast<int>(blockIdx.x) - c_first;
+    const size_t slot_stride = (size_t)p.slot_stride;
+    {
+      float *part = p.partials + (size_t)(c_first + piece + seg) * slot_stride;
+      if (writer) {
+        if (r0 < p.R) {
+#pragma unroll
+          for (int dt = 0; dt < DT; ++dt)
+            *reinterpret_cast<float2 *>(part + (size_t)r0 * D + dt * 8 + colb) = make_float2(o[dt][0], o[dt][1]);
+          if ((lane & 3) == 0) {
+            part[(size_t)p.R * D + r0] = m0;
+            part[(size_t)p.R * D + p.R + r0] = l0;
+          }
+        }
+        if (r1 < p.R) {
+#pragma unroll
+          for (int dt = 0; dt < DT; ++dt)
+            *reinterpret_cast<float2 *>(part + (size_t)r1 * D + dt * 8 + colb) = make_float2(o[dt][2], o[dt][3]);
+          if ((lane & 3) == 0) {
+            part[(size_t)p.R * D + r1] = m1;
+            part[(size_t)p.R * D + p.R + r1] = l1;
+          }
+        }
+      }
+    }
+    __threadfence();
+    __syncthreads();
+    if (tid == 0) {
+      const unsigned prev = atomicAdd(p.tickets + seg, 1u);
+      s_misc[0] = (prev == static_cast<unsigned>(n_pieces - 1)) ? 1 : 0;
+    }
+    __syncthreads();
+    if (s_misc[0]) {
+      // last arrival merges every piece of the segment, in piece order
+      __threadfence();
+      const float *part0 = p.partials + (size_t)(c_first + seg) * slot_stride;
+      for (int idx = tid; idx < p.R * (D / 4); idx += NTHREADS) {
+        const int r = idx / (D / 4), c4 = idx % (D / 4);
+        float M = -INFINITY;
+        for (int q2 = 0; q2 < n_pieces; ++q2)
+          M = fmaxf(M, __ldcg(part0 + q2 * slot_stride + (size_t)p.R * D + r));
+        float lsum = 0.f;
+        float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+        for (int q2 = 0; q2 < n_pieces; ++q2) {
+          const float *pp = part0 + q2 * slot_stride;
+          const float w = exp2f(__ldcg(pp + (size_t)p.R * D + r) - M);
+          lsum += __ldcg(pp + (size_t)p.R * D + p.R + r) * w;
+          const float4 x = __ldcg(reinterpret_cast<const float4 *>(pp + (size_t)r * D) + c4);
+          acc.x += x.x * w; acc.y += x.y * w; acc.z += x.z * w; acc.w += x.w * w;
+        }
+        const float inv = 1.f / lsum;
+        const int i = r / p.group, j = r % p.group;
+        const size_t row = ((size_t)b * p.n_q + i) * p.H_q + (size_t)h_kv * p.group + j;
+        uint2 packed;
+        packed.x = pack_bf16x2(acc.x * inv, acc.y * inv);
+        packed.y = pack_bf16x2(acc.z * inv, acc.w * inv);
+        *reinterpret_cast<uint2 *>(p.out + row * D + 4 * c4) = packed;
+        if (p.lse && c4 == 0) p.lse[row] = (M + log2f(lsum)) * kLn2;
+      }
+      if (tid == 0) p.tickets[seg] = 0u;
+    }
+    __syncthreads();
+  }
+}
+
+// --------------------------------------------------------------------------
+// host side
+// --------------------------------------------------------------------------
+using AttnKernel = void (*)(const CUtensorMap, const CUtensorMap, const AttnParams);
+
+struct AttnVariant {
+  AttnKernel fn;
+  int threads;
+  int stages;
+  int smem_fixed;  // bytes excluding the per-batch arrays
+  int ks, nw;
+};
+
+template <int D, int KS, int NW>
+static AttnVariant make_variant() {
+  constexpr int STAGES = (D == 64) ? 6 : (NW == 4 ? 3 : 5);
+  AttnVariant v;
+  v.fn = verify_attention_kernel<D, KS, NW, STAGES>;
+  v.threads = NW * 32;
+  v.stages = STAGES;
+  v.smem_fixed = AttnSmem<D, STAGES, NW>::bytes(0);
+  v.ks = KS;
+  v.nw = NW;
+  return v;
+}
+
+static AttnVariant select_variant(int D, int R) {
+  const int rt = (R + 15) / 16;
+  if (D == 64) {
+    if (rt == 1) return make_variant<64, 4, 4>();
+    if (rt == 2) return make_variant<64, 2, 4>();
+    if (rt <= 4) return make_variant<64, 1, 4>();
+    return make_variant<64, 1, 8>();
+  }
+  if (rt == 1) return make_variant<128, 4, 4>();
+  if (rt == 2) return make_variant<128, 2, 4>();
+  if (rt <= 4) return make_variant<128, 1, 4>();
+  return make_variant<128, 1, 8>();
+}
+
+struct AttnLayout {
+  size_t tickets_off, partials_off, total;
+};
+
+static AttnLayout attn_layout(int B, int H_kv, int R, int D, long long G) {
+  AttnLayout l;
+  const size_t segs = (size_t)B * H_kv;
+  l.tickets_off = 256;
+  l.partials_off = round_up(l.tickets_off + 4 * segs, 256);
+  l.total = round_up(l.partials_off + (size_t)(G + (long long)segs) * partial_slot_floats(R, D) * 4,
+                     256);
+  return l;
+}
+
+static int check_shapes(int B, int n_q, int H_q, int H_kv, int D, int page_size,
+                        int max_pages_per_seq) {
+  if (B < 1 || B > SF_MAX_BATCH) return fail(SF_ERR_INVALID_ARG, "B=%d outside [1, %d]", B, SF_MAX_BATCH);
+  if (n_q < 1 || n_q > SF_MAX_QUERY_ROWS)
+    return fail(SF_ERR_INVALID_ARG, "n_q=%d outside [1, %d]", n_q, SF_MAX_QUERY_ROWS);
+  if (H_kv < 1 || H_q < 1 || H_q % H_kv != 0)
+    return fail(SF_ERR_INVALID_ARG, "H_q=%d must be a positive multiple of H_kv=%d", H_q, H_kv);
+  if (H_q / H_kv > SF_MAX_GROUP)
+    return fail(SF_ERR_UNSUPPORTED, "group H_q/H_kv=%d above %d", H_q / H_kv, SF_MAX_GROUP);
+  if (D != 64 && D != 128) return fail(SF_ERR_UNSUPPORTED, "head_dim=%d (built: 64, 128)", D);
+  if (page_size != SF_PAGE_SIZE) return fail(SF_ERR_UNSUPPORTED, "page_size=%d (built: 16)", page_size);
+  if (max_pages_per_seq < 1 || (long long)max_pages_per_seq * page_size > (1LL << 30))
+    return fail(SF_ERR_INVALID_ARG, "max_pages_per_seq=%d", max_pages_per_seq);
+  return SF_OK;
+}
+
+struct AttnPlan {
+  AttnVariant v;
+  int G;
+  int smem;
+};
+
+static int plan_attention(int B, int n_q, int H_q, int H_kv, int D, int max_pages_per_seq,
+                          int num_splits, AttnPlan *plan) {
+  DeviceInfo dev;
+  int st = current_device(&dev);
+  if (st != SF_OK) return st;
+  const int R = n_q * (H_q / H_kv);
+  plan->v = select_variant(D, R);
+  plan->smem = plan->v.smem_fixed + 8 * B;
+  if (plan->smem > dev.max_smem_optin)
+    return fail(SF_ERR_UNSUPPORTED, "needs %d B shared memory, device allows %d", plan->smem,
+                dev.max_smem_optin);
+  cudaError_t e = cudaFuncSetAttribute(plan->v.fn, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       plan->smem);
+  if (e != cudaSuccess) return fail(SF_ERR_CUDA, "cudaFuncSetAttribute: %s", cudaGetErrorString(e));
+  const long long max_tiles =
+      (long long)B * H_kv * (((long long)max_pages_per_seq * SF_PAGE_SIZE + kTileTokens - 1) / kTileTokens);
+  long long G = num_splits;
+  if (G <= 0) {
+    int occ = 0;
+    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, plan->v.fn, plan->v.threads, plan->smem);
+    if (e != cudaSuccess) return fail(SF_ERR_CUDA, "occupancy query: %s", cudaGetErrorString(e));
+    G = (long long)dev.sm_count * (occ > 0 ? occ : 1);
+  }
+  if (G > max_tiles) G = max_tiles;
+  if (G > (1 << 20)) G = 1 << 20;
+  plan->G = static_cast<int>(G < 1 ? 1 : G);
+  return SF_OK;
+}
+
+}  // namespace sf
+
+extern "C" {
+
+size_t sf_verify_attention_workspace_size(int B, int n_q, int H_q, int H_kv, int head_dim,
+                                          int max_pages_per_seq, int page_size,
+                                          int num_splits) {
+  if (sf::check_shapes(B, n_q, H_q, H_kv, head_dim, page_size, max_pages_per_seq) != SF_OK)
+    return 0;
+  sf::AttnPlan plan;
+  if (sf::plan_attention(B, n_q, H_q, H_kv, head_dim, max_pages_per_seq, num_splits, &plan) != SF_OK)
+    return 0;
+  return sf::attn_layout(B, H_kv, n_q * (H_q / H_kv), head_dim, plan.G).total;
+}
+
+int sf_verify_attention(const void *q, const void *k_cache, const void *v_cache,
+                        const int32_t *block_table, const int32_t *seq_lens, int B, int n_q,
+                        int H_q, int H_kv, int head_dim, int page_size, int num_pages,
+                        int max_pages_per_seq, float softmax_scale, int num_splits, void *out,
+                        float *lse, void *workspace, size_t workspace_bytes,
+                        cudaStream_t stream) {
+  using namespace sf;
+  clear_error();
+  int st = check_shapes(B, n_q, H_q, H_kv, head_dim, page_size, max_pages_per_seq);
+  if (st != SF_OK) return st;
+  if (!q || !k_cache || !v_cache || !block_table || !seq_lens || !out)
+    return fail(SF_ERR_INVALID_ARG, "a required pointer is NULL");
+  if (num_pages < 1) return fail(SF_ERR_INVALID_ARG, "num_pages=%d", num_pages);
+  if ((long long)num_pages * H_kv * SF_PAGE_SIZE >= (1LL << 31))
+    return fail(SF_ERR_UNSUPPORTED, "KV pool of %d pages x %d heads too large", num_pages, H_kv);
+  if (!aligned(q, 16) || !aligned(k_cache, 16) || !aligned(v_cache, 16) || !aligned(out, 16) ||
+      !aligned(block_table, 4) || !aligned(seq_lens, 4) || (lse && !aligned(lse, 4)))
+    return fail(SF_ERR_INVALID_ARG, "q, caches and out must be 16-byte aligned");
+  if (!(softmax_scale >= 0.f) || std::isinf(softmax_scale))
+    return fail(SF_ERR_INVALID_ARG, "softmax_scale must be finite and >= 0");
+  if (!workspace || !aligned(workspace, 256))
+    return fail(SF_ERR_WORKSPACE, "workspace must be non-NULL and 256-byte aligned");
+
+  AttnPlan plan;
+  st = plan_attention(B, n_q, H_q, H_kv, head_dim, max_pages_per_seq, num_splits, &plan);
+  if (st != SF_OK) return st;
+  const int R = n_q * (H_q / H_kv);
+  const AttnLayout lay = attn_layout(B, H_kv, R, head_dim, plan.G);
+  if (workspace_bytes < lay.total)
+    return fail(SF_ERR_WORKSPACE, "workspace has %zu bytes, needs %zu", workspace_bytes, lay.total);
+
+  const uint64_t rows = (uint64_t)num_pages * H_kv * SF_PAGE_SIZE;
+  CUtensorMap tk, tv;
+  st = encode_tensor_map_2d_bf16(&tk, k_cache, head_dim, rows, (uint64_t)head_dim * 2, 64,
+                                 SF_PAGE_SIZE, true);
+  if (st != SF_OK) return st;
+  st = encode_tensor_map_2d_bf16(&tv, v_cache, head_dim, rows, (uint64_t)head_dim * 2, 64,
+                                 SF_PAGE_SIZE, true);
+  if (st != SF_OK) return st;
+
+  AttnParams prm;
+  uint8_t *ws = static_cast<uint8_t *>(workspace);
+  prm.q = static_cast<const __nv_bfloat16 *>(q);
+  prm.block_table = block_table;
+  prm.seq_lens = seq_lens;
+  prm.out = static_cast<__nv_bfloat16 *>(out);
+  prm.lse = lse;
+  prm.status = reinterpret_cast<uint32_t *>(ws);
+  prm.tickets = reinterpret_cast<uint32_t *>(ws + lay.tickets_off);
+  prm.partials = reinterpret_cast<float *>(ws + lay.partials_off);
+  prm.B = B;
+  prm.n_q = n_q;
+  prm.H_q = H_q;
+  prm.H_kv = H_kv;
+  prm.group = H_q / H_kv;
+  prm.R = R;
+  prm.num_pages = num_pages;
+  prm.max_pages = max_pages_per_seq;
+  prm.max_tokens = max_pages_per_seq * SF_PAGE_SIZE;
+  prm.oob_row = static_cast<int>(rows);
+  const float scale = softmax_scale > 0.f ? softmax_scale : 1.0f / sqrtf((float)head_dim);
+  prm.scale_log2 = scale * 1.4426950408889634f;
+  prm.G = plan.G;
+  prm.slot_stride = partial_slot_floats(R, head_dim);
+
+  plan.v.fn<<<plan.G, plan.v.threads, plan.smem, stream>>>(tk, tv, prm);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return fail(SF_ERR_CUDA, "verify attention launch: %s", cudaGetErrorString(e));
+  return SF_OK;
+}
+
+}  // extern "C"

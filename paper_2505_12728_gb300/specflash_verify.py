@@ -1,0 +1,220 @@
+"""Python binding of the C ABI in include/specflash_verify.h (ctypes).
+
+Argument marshalling only: tensors are checked for dtype, device, shape and
+contiguity, their device pointers and the current CUDA stream are passed to
+the library, and outputs/workspaces are allocated with torch when the caller
+does not supply them.  Every step of the computation runs in the library's
+CUDA kernels; there is no fallback.  If the compiled library is missing the
+first call raises.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import threading
+
+import torch
+
+from . import build_lib
+
+SF_OK = 0
+SF_DEVICE_BAD_PAGE = 0x1
+SF_DEVICE_BAD_TOKEN = 0x2
+SF_DEVICE_TIMEOUT = 0x4
+SF_DEVICE_BAD_SEQLEN = 0x8
+PAGE_SIZE = 16
+
+EXPORTED_SYMBOLS = (
+    "sf_status_string", "sf_last_error", "sf_version", "sf_workspace_init",
+    "sf_read_device_status", "sf_verify_attention_workspace_size", "sf_verify_attention",
+    "sf_accept_workspace_size", "sf_accept",
+)
+
+_lock = threading.Lock()
+_lib = None
+
+
+class SFError(RuntimeError):
+    def __init__(self, status: int, message: str):
+        super().__init__(message)
+        self.status = status
+
+
+def library_path() -> str:
+    return build_lib.LIB
+
+
+def load_library(path: str | None = None):
+    """Load (once) the compiled library; raises if it has not been built."""
+    global _lib
+    with _lock:
+        if _lib is not None:
+            return _lib
+        path = path or library_path()
+        if not os.path.exists(path):
+            raise RuntimeError(
+                f"{path} is missing: build it with paper_2505_12728_gb300.build_lib.build() "
+                "(nvcc for sm_103a); the verification step has no CPU implementation")
+        lib = ctypes.CDLL(path)
+        P, I, F = ctypes.c_void_p, ctypes.c_int, ctypes.c_float
+        S = ctypes.c_size_t
+        lib.sf_status_string.argtypes = [I]
+        lib.sf_status_string.restype = ctypes.c_char_p
+        lib.sf_last_error.argtypes = []
+        lib.sf_last_error.restype = ctypes.c_char_p
+        lib.sf_version.argtypes = []
+        lib.sf_version.restype = I
+        lib.sf_workspace_init.argtypes = [P, S, P]
+        lib.sf_workspace_init.restype = I
+        lib.sf_read_device_status.argtypes = [P, ctypes.POINTER(ctypes.c_uint32)]
+        lib.sf_read_device_status.restype = I
+        lib.sf_verify_attention_workspace_size.argtypes = [I, I, I, I, I, I, I, I]
+        lib.sf_verify_attention_workspace_size.restype = S
+        lib.sf_verify_attention.argtypes = [P, P, P, P, P, I, I, I, I, I, I, I, I, F, I, P, P, P,
+                                            S, P]
+        lib.sf_verify_attention.restype = I
+        lib.sf_accept_workspace_size.argtypes = [I, I, I]
+        lib.sf_accept_workspace_size.restype = S
+        lib.sf_accept.argtypes = [P, P, P, P, P, I, I, I, P, P, P, P, S, P]
+        lib.sf_accept.restype = I
+        _lib = lib
+        return lib
+
+
+def _check(status: int):
+    if status != SF_OK:
+        lib = load_library()
+        raise SFError(status, f"{lib.sf_status_string(status).decode()}: "
+                              f"{lib.sf_last_error().decode()}")
+
+
+def _ptr(t):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def _stream_handle(stream):
+    s = torch.cuda.current_stream() if stream is None else stream
+    return ctypes.c_void_p(s.cuda_stream)
+
+
+def _need(t, name, dtype, shape=None):
+    if not isinstance(t, torch.Tensor):
+        raise TypeError(f"{name} must be a torch.Tensor")
+    if t.dtype != dtype:
+        raise TypeError(f"{name} must be {dtype}, got {t.dtype}")
+    if not t.is_cuda:
+        raise ValueError(f"{name} must be a CUDA tensor")
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+    if shape is not None and tuple(t.shape) != tuple(shape):
+        raise ValueError(f"{name} has shape {tuple(t.shape)}, expected {tuple(shape)}")
+
+
+# --------------------------------------------------------------------------- #
+# workspaces                                                                  #
+# --------------------------------------------------------------------------- #
+def verify_attention_workspace_size(B, n_q, H_q, H_kv, head_dim, max_pages_per_seq,
+                                    page_size=PAGE_SIZE, num_splits=0) -> int:
+    n = load_library().sf_verify_attention_workspace_size(B, n_q, H_q, H_kv, head_dim,
+                                                          max_pages_per_seq, page_size,
+                                                          num_splits)
+    if n == 0:
+        raise SFError(1, "invalid verify-attention shape: " + load_library().sf_last_error().decode())
+    return int(n)
+
+
+def accept_workspace_size(B, k, V) -> int:
+    n = load_library().sf_accept_workspace_size(B, k, V)
+    if n == 0:
+        raise SFError(1, "invalid acceptance shape: " + load_library().sf_last_error().decode())
+    return int(n)
+
+
+def new_workspace(nbytes: int, device=None) -> torch.Tensor:
+    """A zero-filled uint8 device buffer (the library's counters start at 0)."""
+    return torch.zeros(int(nbytes), dtype=torch.uint8, device=device or "cuda")
+
+
+def workspace_init(workspace: torch.Tensor, stream=None):
+    _check(load_library().sf_workspace_init(_ptr(workspace), workspace.numel(),
+                                            _stream_handle(stream)))
+
+
+def read_device_status(workspace: torch.Tensor) -> int:
+    v = ctypes.c_uint32(0)
+    _check(load_library().sf_read_device_status(_ptr(workspace), ctypes.byref(v)))
+    return int(v.value)
+
+
+# --------------------------------------------------------------------------- #
+# verification attention                                                      #
+# --------------------------------------------------------------------------- #
+def verify_attention(q, k_cache, v_cache, block_table, seq_lens, *, out=None, lse=None,
+                     workspace=None, softmax_scale=0.0, num_splits=0, stream=None,
+                     with_lse=True):
+    """sf_verify_attention: q bf16 [B][n_q][H_q][d]; k/v_cache bf16
+    [pages][H_kv][16][d]; block_table int32 [B][max_pages]; seq_lens int32 [B]
+    (prefix + n_q).  Returns (out bf16 [B][n_q][H_q][d], lse fp32 [B][n_q][H_q]
+    or None)."""
+    B, n_q, H_q, d = q.shape
+    num_pages, H_kv, page, d2 = k_cache.shape
+    _need(q, "q", torch.bfloat16)
+    _need(k_cache, "k_cache", torch.bfloat16)
+    _need(v_cache, "v_cache", torch.bfloat16, k_cache.shape)
+    _need(block_table, "block_table", torch.int32)
+    _need(seq_lens, "seq_lens", torch.int32, (B,))
+    if d2 != d:
+        raise ValueError("head_dim of q and caches differ")
+    max_pages = block_table.shape[1]
+    if out is None:
+        out = torch.empty_like(q)
+    _need(out, "out", torch.bfloat16, q.shape)
+    if lse is None and with_lse:
+        lse = torch.empty((B, n_q, H_q), dtype=torch.float32, device=q.device)
+    if lse is not None:
+        _need(lse, "lse", torch.float32, (B, n_q, H_q))
+    if workspace is None:
+        workspace = new_workspace(verify_attention_workspace_size(
+            B, n_q, H_q, H_kv, d, max_pages, page, num_splits), q.device)
+    _check(load_library().sf_verify_attention(
+        _ptr(q), _ptr(k_cache), _ptr(v_cache), _ptr(block_table), _ptr(seq_lens), B, n_q, H_q,
+        H_kv, d, page, num_pages, max_pages, float(softmax_scale), int(num_splits), _ptr(out),
+        _ptr(lse), _ptr(workspace), workspace.numel(), _stream_handle(stream)))
+    return out, lse
+
+
+# --------------------------------------------------------------------------- #
+# acceptance                                                                  #
+# --------------------------------------------------------------------------- #
+def accept(target_logits, draft_probs, draft_tokens, uniforms, temperature, *,
+           num_accepted=None, out_tokens=None, accept_ratio=None, workspace=None, stream=None,
+           with_ratio=True):
+    """sf_accept: target_logits fp32 [B][k+1][V], draft_probs fp32 [B][k][V],
+    draft_tokens int32 [B][k], uniforms fp32 [B][k+1], temperature fp32 [B]
+    (<= 0 greedy).  Returns (num_accepted int32 [B], out_tokens int32 [B][k+1],
+    accept_ratio fp32 [B][k] or None)."""
+    B, k1, V = target_logits.shape
+    k = k1 - 1
+    _need(target_logits, "target_logits", torch.float32)
+    _need(draft_probs, "draft_probs", torch.float32, (B, k, V))
+    _need(draft_tokens, "draft_tokens", torch.int32, (B, k))
+    _need(uniforms, "uniforms", torch.float32, (B, k + 1))
+    _need(temperature, "temperature", torch.float32, (B,))
+    dev = target_logits.device
+    if num_accepted is None:
+        num_accepted = torch.empty(B, dtype=torch.int32, device=dev)
+    if out_tokens is None:
+        out_tokens = torch.empty((B, k + 1), dtype=torch.int32, device=dev)
+    if accept_ratio is None and with_ratio:
+        accept_ratio = torch.empty((B, k), dtype=torch.float32, device=dev)
+    _need(num_accepted, "num_accepted", torch.int32, (B,))
+    _need(out_tokens, "out_tokens", torch.int32, (B, k + 1))
+    if accept_ratio is not None:
+        _need(accept_ratio, "accept_ratio", torch.float32, (B, k))
+    if workspace is None:
+        workspace = new_workspace(accept_workspace_size(B, k, V), dev)
+    _check(load_library().sf_accept(
+        _ptr(target_logits), _ptr(draft_probs), _ptr(draft_tokens), _ptr(uniforms),
+        _ptr(temperature), B, k, V, _ptr(num_accepted), _ptr(out_tokens), _ptr(accept_ratio),
+        _ptr(workspace), workspace.numel(), _stream_handle(stream)))
+    return num_accepted, out_tokens, accept_ratio
