@@ -128,6 +128,35 @@ int sf_verify_attention(const void *q, const void *k_cache, const void *v_cache,
                         cudaStream_t stream);
 
 /* ------------------------------------------------------------------------ */
+/* Verification attention without a caller workspace.  The paper has no      */
+/* counterpart: this is a deployment convenience of this library.            */
+/*                                                                           */
+/* For callers that cannot allocate device memory when they verify: a        */
+/* serving runtime whose memory manager owns the whole device and refuses    */
+/* allocations mid-request, a plug-in that receives only its input and       */
+/* output buffers, or a runtime with a memory budget fixed before serving.   */
+/* Same arguments and results as sf_verify_attention, minus the workspace:   */
+/* the library uses its own scratch, a 16 MiB device array that exists on    */
+/* every GPU that loads the library until the process exits.  Shapes whose   */
+/* workspace (sf_verify_attention_workspace_size) exceeds 16 MiB are         */
+/* rejected with SF_ERR_UNSUPPORTED before anything is enqueued.             */
+/* The call allocates nothing: it clears the scratch's counters with         */
+/* cudaMemsetAsync on `stream`, then launches the kernel.                    */
+/* Its first call on a device looks up the scratch's device address (once    */
+/* per device, cached); make that first call before any stream capture.      */
+/* All calls share the one scratch array, which keeps the previous call's    */
+/* contents: calls that may overlap on the GPU (different streams, or        */
+/* threads without ordering) race and give wrong results; serialise them.    */
+/* Device data errors never fault here either, but their status bits stay   */
+/* in the library's scratch; use sf_verify_attention to read them.           */
+/* ------------------------------------------------------------------------ */
+int sf_verify_attention_noalloc(const void *q, const void *k_cache, const void *v_cache,
+                                const int32_t *block_table, const int32_t *seq_lens, int B,
+                                int n_q, int H_q, int H_kv, int head_dim, int page_size,
+                                int num_pages, int max_pages_per_seq, float softmax_scale,
+                                int num_splits, void *out, float *lse, cudaStream_t stream);
+
+/* ------------------------------------------------------------------------ */
 /* Acceptance (Sec. 3.1: acceptance probability as the ratio of target to    */
 /* draft probability, discard from the first rejection on, resample from the */
 /* residual distribution; Sec. 3.3: "the standard token-wise acceptance-     */

@@ -766,3 +766,79 @@ int sf_verify_attention(const void *q, const void *k_cache, const void *v_cache,
 }
 
 }  // extern "C"
+
+// --------------------------------------------------------------------------
+// Verification attention without a caller workspace.
+//
+// Some callers cannot allocate device memory at the point where they run the
+// verification step: an inference server whose memory manager owns every
+// byte of the device and refuses allocations while serving, a plug-in that
+// is handed only its input and output buffers, or a runtime that pre-plans a
+// fixed memory budget before the first request.  For them the library keeps
+// its own scratch: one file-scope device array, created with the module on
+// every GPU that loads this library and held until the process exits.  The
+// entry point below runs the same kernel as sf_verify_attention with that
+// array as its workspace, after clearing the part that must start at zero.
+// --------------------------------------------------------------------------
+namespace sf {
+
+constexpr size_t kStaticScratchBytes = size_t(16) << 20;  // 16 MiB per device
+
+static __device__ __align__(256) uint8_t g_static_scratch[kStaticScratchBytes];
+
+// Device address of g_static_scratch on the current device.  Host code must
+// not use the symbol itself (it is a host-side stand-in, not a device
+// address); the address is looked up once per device, with that device
+// current, and cached.
+static int static_scratch_address(void **out) {
+  static std::mutex mu;
+  static void *addr[64] = {nullptr};
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return fail(SF_ERR_CUDA, "cudaGetDevice: %s", cudaGetErrorString(e));
+  if (dev < 0 || dev >= 64) return fail(SF_ERR_UNSUPPORTED, "device ordinal %d", dev);
+  std::lock_guard<std::mutex> lock(mu);
+  if (!addr[dev]) {
+    void *p = nullptr;
+    e = cudaGetSymbolAddress(&p, g_static_scratch);
+    if (e != cudaSuccess || !p)
+      return fail(SF_ERR_CUDA, "cudaGetSymbolAddress(scratch): %s", cudaGetErrorString(e));
+    addr[dev] = p;
+  }
+  *out = addr[dev];
+  return SF_OK;
+}
+
+}  // namespace sf
+
+extern "C" int sf_verify_attention_noalloc(const void *q, const void *k_cache,
+                                           const void *v_cache, const int32_t *block_table,
+                                           const int32_t *seq_lens, int B, int n_q, int H_q,
+                                           int H_kv, int head_dim, int page_size, int num_pages,
+                                           int max_pages_per_seq, float softmax_scale,
+                                           int num_splits, void *out, float *lse,
+                                           cudaStream_t stream) {
+  using namespace sf;
+  clear_error();
+  int st = check_shapes(B, n_q, H_q, H_kv, head_dim, page_size, max_pages_per_seq);
+  if (st != SF_OK) return st;
+  AttnPlan plan;
+  st = plan_attention(B, n_q, H_q, H_kv, head_dim, max_pages_per_seq, num_splits, &plan);
+  if (st != SF_OK) return st;
+  const AttnLayout lay = attn_layout(B, H_kv, n_q * (H_q / H_kv), head_dim, plan.G);
+  if (lay.total > kStaticScratchBytes)
+    return fail(SF_ERR_UNSUPPORTED,
+                "this shape needs %zu bytes of scratch but the built-in scratch holds %zu; "
+                "use sf_verify_attention with a caller workspace (or a smaller num_splits)",
+                lay.total, kStaticScratchBytes);
+  void *scratch = nullptr;
+  st = static_scratch_address(&scratch);
+  if (st != SF_OK) return st;
+  // The status word and the merge tickets must start at zero; the partials
+  // need no clearing.  The scratch keeps whatever the previous call left.
+  cudaError_t e = cudaMemsetAsync(scratch, 0, lay.partials_off, stream);
+  if (e != cudaSuccess) return fail(SF_ERR_CUDA, "clearing the scratch: %s", cudaGetErrorString(e));
+  return sf_verify_attention(q, k_cache, v_cache, block_table, seq_lens, B, n_q, H_q, H_kv,
+                             head_dim, page_size, num_pages, max_pages_per_seq, softmax_scale,
+                             num_splits, out, lse, scratch, kStaticScratchBytes, stream);
+}

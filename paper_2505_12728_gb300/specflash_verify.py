@@ -27,6 +27,7 @@ PAGE_SIZE = 16
 EXPORTED_SYMBOLS = (
     "sf_status_string", "sf_last_error", "sf_version", "sf_workspace_init",
     "sf_read_device_status", "sf_verify_attention_workspace_size", "sf_verify_attention",
+    "sf_verify_attention_noalloc",
     "sf_accept_workspace_size", "sf_accept",
 )
 
@@ -73,6 +74,9 @@ def load_library(path: str | None = None):
         lib.sf_verify_attention.argtypes = [P, P, P, P, P, I, I, I, I, I, I, I, I, F, I, P, P, P,
                                             S, P]
         lib.sf_verify_attention.restype = I
+        lib.sf_verify_attention_noalloc.argtypes = [P, P, P, P, P, I, I, I, I, I, I, I, I, F, I,
+                                                    P, P, P]
+        lib.sf_verify_attention_noalloc.restype = I
         lib.sf_accept_workspace_size.argtypes = [I, I, I]
         lib.sf_accept_workspace_size.restype = S
         lib.sf_accept.argtypes = [P, P, P, P, P, I, I, I, P, P, P, P, S, P]
@@ -180,6 +184,34 @@ def verify_attention(q, k_cache, v_cache, block_table, seq_lens, *, out=None, ls
         _ptr(q), _ptr(k_cache), _ptr(v_cache), _ptr(block_table), _ptr(seq_lens), B, n_q, H_q,
         H_kv, d, page, num_pages, max_pages, float(softmax_scale), int(num_splits), _ptr(out),
         _ptr(lse), _ptr(workspace), workspace.numel(), _stream_handle(stream)))
+    return out, lse
+
+
+def verify_attention_noalloc(q, k_cache, v_cache, block_table, seq_lens, *, out=None, lse=None,
+                             softmax_scale=0.0, num_splits=0, stream=None, with_lse=True):
+    """sf_verify_attention_noalloc: the same computation as verify_attention
+    for callers that cannot allocate device memory while verifying; the
+    library's own 16 MiB device scratch replaces the workspace (calls that
+    overlap on the GPU race on it).  Outputs may still be allocated here when
+    not supplied."""
+    B, n_q, H_q, d = q.shape
+    num_pages, H_kv, page, _ = k_cache.shape
+    _need(q, "q", torch.bfloat16)
+    _need(k_cache, "k_cache", torch.bfloat16)
+    _need(v_cache, "v_cache", torch.bfloat16, k_cache.shape)
+    _need(block_table, "block_table", torch.int32)
+    _need(seq_lens, "seq_lens", torch.int32, (B,))
+    if out is None:
+        out = torch.empty_like(q)
+    _need(out, "out", torch.bfloat16, q.shape)
+    if lse is None and with_lse:
+        lse = torch.empty((B, n_q, H_q), dtype=torch.float32, device=q.device)
+    if lse is not None:
+        _need(lse, "lse", torch.float32, (B, n_q, H_q))
+    _check(load_library().sf_verify_attention_noalloc(
+        _ptr(q), _ptr(k_cache), _ptr(v_cache), _ptr(block_table), _ptr(seq_lens), B, n_q, H_q,
+        H_kv, d, page, num_pages, block_table.shape[1], float(softmax_scale), int(num_splits),
+        _ptr(out), _ptr(lse), _stream_handle(stream)))
     return out, lse
 
 
