@@ -119,6 +119,18 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
   return *reinterpret_cast<uint32_t *>(&v);
 }
 
+// Programmatic dependent launch: allow the next kernel on the stream to be
+// scheduled now (it still waits for this grid before using its results) ...
+__device__ __forceinline__ void grid_launch_dependents() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
+// ... and wait until the previous kernel on the stream has completed and its
+// memory operations are visible (a no-op when launched without the attribute).
+__device__ __forceinline__ void grid_dependency_wait() {
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+}
+
 __device__ __forceinline__ void set_status(uint32_t *status, uint32_t bits) {
   atomicOr(status, bits);
 }

@@ -33,7 +33,9 @@
 //    loaded as zero boxes (TMA out-of-bounds fill); bad indices set a bit in
 //    the status word.  Every mbarrier wait is bounded.
 #include <cmath>
+#include <map>
 #include <mutex>
+#include <tuple>
 
 #include "sf_device.cuh"
 #include "sf_host.h"
@@ -54,7 +56,9 @@ struct AttnParams {
   __nv_bfloat16 *out;
   float *lse;
   uint32_t *status;
-  uint32_t *tickets;  // [B * H_kv]
+  int2 *seg_desc;     // [B * H_kv]: {first CTA, pieces} of each segment
+  uint32_t *tickets;  // [B * H_kv], zero between calls (in-kernel merge)
+  int merge_in_kernel;  // 1: last CTA of a segment merges; 0: merge kernel
   float *partials;    // [G + B * H_kv][R][D + 2]
   int B, n_q, H_q, H_kv, group, R;
   int num_pages, max_pages, max_tokens;
@@ -139,6 +143,58 @@ __device__ __forceinline__ int owner_cta(long long t, long long Tot, int G) {
   return static_cast<int>(((t + 1) * G - 1) / Tot);
 }
 
+constexpr int kMergeBatch = 16;
+
+template <bool kBypassL1, typename T>
+__device__ __forceinline__ T merge_load(const T *p) {
+  if constexpr (kBypassL1) return __ldcg(p);
+  else return *p;
+}
+
+// Combines the pieces of one output (row r, columns 4*c4 .. 4*c4+3) of a
+// split segment, in piece order:
+//   M = max_q m_q,  L = sum_q l_q 2^(m_q - M),  O = sum_q 2^(m_q - M) O_q / L.
+// The pieces are read in batches of kMergeBatch with an online rescale; all
+// loads of a batch are issued before any is used, so a batch costs one
+// memory round trip.  Partial slot layout: O [R][D], m [R], l [R].
+template <int D, bool kBypassL1>
+__device__ __forceinline__ void merge_one(const float *part0, size_t stride, int R, int r, int c4,
+                                          int n_pieces, float4 &o, float &M, float &Ls) {
+  const float *mrow = part0 + (size_t)R * D + r;
+  const float *lrow = mrow + R;
+  const float4 *orow = reinterpret_cast<const float4 *>(part0 + (size_t)r * D) + c4;
+  const size_t stride4 = stride / 4;
+  M = -INFINITY;
+  Ls = 0.f;
+  float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+  for (int q0 = 0; q0 < n_pieces; q0 += kMergeBatch) {
+    float mv[kMergeBatch], lv[kMergeBatch];
+    float4 xv[kMergeBatch];
+#pragma unroll
+    for (int u = 0; u < kMergeBatch; ++u) {
+      const bool in = q0 + u < n_pieces;
+      mv[u] = in ? merge_load<kBypassL1>(mrow + (q0 + u) * stride) : -INFINITY;
+      lv[u] = in ? merge_load<kBypassL1>(lrow + (q0 + u) * stride) : 0.f;
+      xv[u] = in ? merge_load<kBypassL1>(orow + (q0 + u) * stride4) : make_float4(0.f, 0.f, 0.f, 0.f);
+    }
+    float Mb = M;
+#pragma unroll
+    for (int u = 0; u < kMergeBatch; ++u) Mb = fmaxf(Mb, mv[u]);
+    const float a = exp2f(M - Mb);  // first batch: M = -inf, a = 0
+    Ls *= a;
+    acc.x *= a; acc.y *= a; acc.z *= a; acc.w *= a;
+#pragma unroll
+    for (int u = 0; u < kMergeBatch; ++u) {
+      const float w = exp2f(mv[u] - Mb);
+      Ls += lv[u] * w;
+      acc.x += xv[u].x * w; acc.y += xv[u].y * w; acc.z += xv[u].z * w; acc.w += xv[u].w * w;
+    }
+    M = Mb;
+  }
+  const float inv = 1.f / Ls;
+  o = make_float4(acc.x * inv, acc.y * inv, acc.z * inv, acc.w * inv);
+}
+
 template <int D, int KS, int NW, int STAGES>
 __global__ void __launch_bounds__(NW * 32, (NW == 4 ? 2 : 1))
 verify_attention_kernel(const __grid_constant__ CUtensorMap tmap_k,
@@ -168,6 +224,12 @@ verify_attention_kernel(const __grid_constant__ CUtensorMap tmap_k,
   const int row_tiles = (p.R + 15) >> 4;
   const bool active = rt < row_tiles;
 
+  // Let the next kernel on the stream be scheduled as CTAs of this grid
+  // finish.  Work that does not depend on the previous kernel on
+  // the stream (barrier set-up, the tile partition, block-table reads and the
+  // first K/V copies) runs before grid_dependency_wait(); Q is read and
+  // results are written only after it.
+  grid_launch_dependents();
   if (tid == 0) {
     for (int s = 0; s < STAGES; ++s) mbar_init(bar0 + 8 * s, 1);
     fence_mbar_init();
@@ -188,6 +250,7 @@ verify_attention_kernel(const __grid_constant__ CUtensorMap tmap_k,
   const long long t_end = (long long)(blockIdx.x + 1) * Tot / G;
 
   const uint64_t policy = l2_policy_evict_first();
+  bool waited = false;    // grid_dependency_wait() done
   uint32_t consumed = 0;  // tiles consumed by this CTA so far (ring position)
   bool timed_out = false;
 
@@ -249,6 +312,12 @@ verify_attention_kernel(const __grid_constant__ CUtensorMap tmap_k,
       }
       if (lane < kPagesPerTile && prologue < n_tiles) next_phys = fetch_page(lt0 + prologue, lane);
     }
+
+    if (!waited) {
+      grid_dependency_wait();
+      waited = true;
+    }
+    if (lt0 == 0 && tid == 0) p.seg_desc[seg] = make_int2(c_first, n_pieces);
 
     // ---- consumers: Q fragments of this warp's 16 rows ----
     // row r = i * g + j  <->  (draft row i, query head h_kv * g + j)
@@ -508,11 +577,10 @@ verify_attention_kernel(const __grid_constant__ CUtensorMap tmap_k,
       continue;
     }
 
-    // ---- several pieces: write this piece's partial, take a ticket ----
-    const int piece = static_cast<int>(blockIdx.x) - c_first;
-    const size_t slot_stride = (size_t)p.slot_stride;
+    // ---- several pieces: write this piece's partial ----
+    const size_t stride = (size_t)p.slot_stride;
     {
-      float *part = p.partials + (size_t)(c_first + piece + seg) * slot_stride;
+      float *part = p.partials + (size_t)(blockIdx.x + seg) * stride;
       if (writer) {
         if (r0 < p.R) {
 #pragma unroll
@@ -534,6 +602,9 @@ verify_attention_kernel(const __grid_constant__ CUtensorMap tmap_k,
         }
       }
     }
+    if (!p.merge_in_kernel) continue;  // verify_merge_kernel combines the pieces
+
+    // ---- few rows: the last CTA of the segment to finish merges it ----
     __threadfence();
     __syncthreads();
     if (tid == 0) {
@@ -542,36 +613,66 @@ verify_attention_kernel(const __grid_constant__ CUtensorMap tmap_k,
     }
     __syncthreads();
     if (s_misc[0]) {
-      // last arrival merges every piece of the segment, in piece order
+      // every piece is written: this CTA merges the segment
       __threadfence();
-      const float *part0 = p.partials + (size_t)(c_first + seg) * slot_stride;
+      const float *part0 = p.partials + (size_t)(c_first + seg) * stride;
       for (int idx = tid; idx < p.R * (D / 4); idx += NTHREADS) {
         const int r = idx / (D / 4), c4 = idx % (D / 4);
-        float M = -INFINITY;
-        for (int q2 = 0; q2 < n_pieces; ++q2)
-          M = fmaxf(M, __ldcg(part0 + q2 * slot_stride + (size_t)p.R * D + r));
-        float lsum = 0.f;
-        float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-        for (int q2 = 0; q2 < n_pieces; ++q2) {
-          const float *pp = part0 + q2 * slot_stride;
-          const float w = exp2f(__ldcg(pp + (size_t)p.R * D + r) - M);
-          lsum += __ldcg(pp + (size_t)p.R * D + p.R + r) * w;
-          const float4 x = __ldcg(reinterpret_cast<const float4 *>(pp + (size_t)r * D) + c4);
-          acc.x += x.x * w; acc.y += x.y * w; acc.z += x.z * w; acc.w += x.w * w;
-        }
-        const float inv = 1.f / lsum;
+        float4 ov;
+        float M, Ls;
+        merge_one<D, true>(part0, stride, p.R, r, c4, n_pieces, ov, M, Ls);
         const int i = r / p.group, j = r % p.group;
         const size_t row = ((size_t)b * p.n_q + i) * p.H_q + (size_t)h_kv * p.group + j;
         uint2 packed;
-        packed.x = pack_bf16x2(acc.x * inv, acc.y * inv);
-        packed.y = pack_bf16x2(acc.z * inv, acc.w * inv);
+        packed.x = pack_bf16x2(ov.x, ov.y);
+        packed.y = pack_bf16x2(ov.z, ov.w);
         *reinterpret_cast<uint2 *>(p.out + row * D + 4 * c4) = packed;
-        if (p.lse && c4 == 0) p.lse[row] = (M + log2f(lsum)) * kLn2;
+        if (p.lse && c4 == 0) p.lse[row] = (M + log2f(Ls)) * kLn2;
       }
       if (tid == 0) p.tickets[seg] = 0u;
     }
     __syncthreads();
   }
+}
+
+// Merge for shapes with many rows per KV head (GQA): the pieces of every
+// split segment are combined by a grid over (row groups, segments), one
+// thread per 4 output columns of a row, in piece order (deterministic):
+//   M = max_q m_q,  L = sum_q l_q 2^(m_q - M),  O = sum_q 2^(m_q - M) O_q / L,
+//   lse = (M + log2 L) ln 2.
+// Pieces are read in batches of kMergeBatch with a running (online) rescale,
+// so a batch costs one memory round trip.  Launched right after the split
+// kernel with programmatic stream serialisation: its CTAs may be scheduled
+// while the split grid drains, and wait for it before reading anything.
+constexpr int kMergeThreads = 128;
+
+template <int D>
+__global__ void __launch_bounds__(kMergeThreads)
+verify_merge_kernel(const __grid_constant__ AttnParams p) {
+  constexpr float kLn2 = 0.6931471805599453f;
+  constexpr int C4 = D / 4;                       // threads per row
+  constexpr int RPC = kMergeThreads / C4;         // rows per CTA
+  grid_launch_dependents();
+  grid_dependency_wait();
+  const int seg = blockIdx.y;
+  const int2 desc = p.seg_desc[seg];              // {first CTA, pieces}
+  if (desc.y <= 1) return;                        // the split kernel wrote it
+  const int r = blockIdx.x * RPC + threadIdx.x / C4;
+  const int c4 = threadIdx.x % C4;
+  if (r >= p.R) return;
+  const size_t stride = (size_t)p.slot_stride;
+  float4 ov;
+  float M, Ls;
+  merge_one<D, false>(p.partials + (size_t)(desc.x + seg) * stride, stride, p.R, r, c4, desc.y,
+                      ov, M, Ls);
+  const int b = seg / p.H_kv, h_kv = seg % p.H_kv;
+  const int i = r / p.group, j = r % p.group;
+  const size_t row = ((size_t)b * p.n_q + i) * p.H_q + (size_t)h_kv * p.group + j;
+  uint2 packed;
+  packed.x = pack_bf16x2(ov.x, ov.y);
+  packed.y = pack_bf16x2(ov.z, ov.w);
+  *reinterpret_cast<uint2 *>(p.out + row * D + 4 * c4) = packed;
+  if (p.lse && c4 == 0) p.lse[row] = (M + log2f(Ls)) * kLn2;
 }
 
 // --------------------------------------------------------------------------
@@ -615,13 +716,14 @@ static AttnVariant select_variant(int D, int R) {
 }
 
 struct AttnLayout {
-  size_t tickets_off, partials_off, total;
+  size_t desc_off, tickets_off, partials_off, total;
 };
 
 static AttnLayout attn_layout(int B, int H_kv, int R, int D, long long G) {
   AttnLayout l;
   const size_t segs = (size_t)B * H_kv;
-  l.tickets_off = 256;
+  l.desc_off = 256;
+  l.tickets_off = round_up(l.desc_off + 8 * segs, 256);
   l.partials_off = round_up(l.tickets_off + 4 * segs, 256);
   l.total = round_up(l.partials_off + (size_t)(G + (long long)segs) * partial_slot_floats(R, D) * 4,
                      256);
@@ -650,6 +752,32 @@ struct AttnPlan {
   int smem;
 };
 
+// Per-device, per-kernel launch facts, computed once: the dynamic shared
+// memory limit is raised to the largest size any batch needs, and resident
+// CTAs per SM are cached per shared-memory size.
+static int kernel_setup(const AttnVariant &v, int dev, int smem, int *occ_out) {
+  static std::mutex mu;
+  static std::map<std::tuple<void *, int, int>, int> occ_cache;
+  static std::map<std::pair<void *, int>, bool> attr_done;
+  std::lock_guard<std::mutex> lock(mu);
+  void *key = reinterpret_cast<void *>(v.fn);
+  if (!attr_done[{key, dev}]) {
+    cudaError_t e = cudaFuncSetAttribute(v.fn, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         v.smem_fixed + 8 * SF_MAX_BATCH);
+    if (e != cudaSuccess) return fail(SF_ERR_CUDA, "cudaFuncSetAttribute: %s", cudaGetErrorString(e));
+    attr_done[{key, dev}] = true;
+  }
+  auto it = occ_cache.find({key, dev, smem});
+  if (it == occ_cache.end()) {
+    int occ = 0;
+    cudaError_t e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, v.fn, v.threads, smem);
+    if (e != cudaSuccess) return fail(SF_ERR_CUDA, "occupancy query: %s", cudaGetErrorString(e));
+    it = occ_cache.emplace(std::make_tuple(key, dev, smem), occ > 0 ? occ : 1).first;
+  }
+  *occ_out = it->second;
+  return SF_OK;
+}
+
 static int plan_attention(int B, int n_q, int H_q, int H_kv, int D, int max_pages_per_seq,
                           int num_splits, AttnPlan *plan) {
   DeviceInfo dev;
@@ -658,24 +786,40 @@ static int plan_attention(int B, int n_q, int H_q, int H_kv, int D, int max_page
   const int R = n_q * (H_q / H_kv);
   plan->v = select_variant(D, R);
   plan->smem = plan->v.smem_fixed + 8 * B;
-  if (plan->smem > dev.max_smem_optin)
-    return fail(SF_ERR_UNSUPPORTED, "needs %d B shared memory, device allows %d", plan->smem,
-                dev.max_smem_optin);
-  cudaError_t e = cudaFuncSetAttribute(plan->v.fn, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       plan->smem);
-  if (e != cudaSuccess) return fail(SF_ERR_CUDA, "cudaFuncSetAttribute: %s", cudaGetErrorString(e));
+  if (plan->v.smem_fixed + 8 * SF_MAX_BATCH > dev.max_smem_optin)
+    return fail(SF_ERR_UNSUPPORTED, "needs %d B shared memory, device allows %d",
+                plan->v.smem_fixed + 8 * SF_MAX_BATCH, dev.max_smem_optin);
+  int occ = 1;
+  st = kernel_setup(plan->v, dev.ordinal, plan->smem, &occ);
+  if (st != SF_OK) return st;
   const long long max_tiles =
       (long long)B * H_kv * (((long long)max_pages_per_seq * SF_PAGE_SIZE + kTileTokens - 1) / kTileTokens);
-  long long G = num_splits;
-  if (G <= 0) {
-    int occ = 0;
-    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, plan->v.fn, plan->v.threads, plan->smem);
-    if (e != cudaSuccess) return fail(SF_ERR_CUDA, "occupancy query: %s", cudaGetErrorString(e));
-    G = (long long)dev.sm_count * (occ > 0 ? occ : 1);
-  }
+  long long G = num_splits > 0 ? num_splits : (long long)dev.sm_count * occ;
   if (G > max_tiles) G = max_tiles;
   if (G > (1 << 20)) G = 1 << 20;
   plan->G = static_cast<int>(G < 1 ? 1 : G);
+  return SF_OK;
+}
+
+// TMA descriptors of the K and V caches, cached by (address, rows, head_dim)
+// so that repeated calls on the same caches skip the encoding.
+static int cache_tensor_map(CUtensorMap *out, const void *base, uint64_t rows, int head_dim) {
+  static std::mutex mu;
+  static std::map<std::tuple<const void *, uint64_t, int>, CUtensorMap> maps;
+  {
+    std::lock_guard<std::mutex> lock(mu);
+    auto it = maps.find({base, rows, head_dim});
+    if (it != maps.end()) {
+      *out = it->second;
+      return SF_OK;
+    }
+  }
+  int st = encode_tensor_map_2d_bf16(out, base, head_dim, rows, (uint64_t)head_dim * 2, 64,
+                                     SF_PAGE_SIZE, true);
+  if (st != SF_OK) return st;
+  std::lock_guard<std::mutex> lock(mu);
+  if (maps.size() >= 4096) maps.clear();
+  maps.emplace(std::make_tuple(base, rows, head_dim), *out);
   return SF_OK;
 }
 
@@ -727,11 +871,9 @@ int sf_verify_attention(const void *q, const void *k_cache, const void *v_cache,
 
   const uint64_t rows = (uint64_t)num_pages * H_kv * SF_PAGE_SIZE;
   CUtensorMap tk, tv;
-  st = encode_tensor_map_2d_bf16(&tk, k_cache, head_dim, rows, (uint64_t)head_dim * 2, 64,
-                                 SF_PAGE_SIZE, true);
+  st = cache_tensor_map(&tk, k_cache, rows, head_dim);
   if (st != SF_OK) return st;
-  st = encode_tensor_map_2d_bf16(&tv, v_cache, head_dim, rows, (uint64_t)head_dim * 2, 64,
-                                 SF_PAGE_SIZE, true);
+  st = cache_tensor_map(&tv, v_cache, rows, head_dim);
   if (st != SF_OK) return st;
 
   AttnParams prm;
@@ -742,7 +884,12 @@ int sf_verify_attention(const void *q, const void *k_cache, const void *v_cache,
   prm.out = static_cast<__nv_bfloat16 *>(out);
   prm.lse = lse;
   prm.status = reinterpret_cast<uint32_t *>(ws);
+  prm.seg_desc = reinterpret_cast<int2 *>(ws + lay.desc_off);
   prm.tickets = reinterpret_cast<uint32_t *>(ws + lay.tickets_off);
+  // One row tile (MHA, n_q <= 16): the partials are small and the last CTA
+  // of a segment merges them without a second launch.  More rows (GQA): a
+  // grid-wide merge kernel spreads the larger partials over many SMs.
+  prm.merge_in_kernel = R <= 16 ? 1 : 0;
   prm.partials = reinterpret_cast<float *>(ws + lay.partials_off);
   prm.B = B;
   prm.n_q = n_q;
@@ -759,9 +906,29 @@ int sf_verify_attention(const void *q, const void *k_cache, const void *v_cache,
   prm.G = plan.G;
   prm.slot_stride = partial_slot_floats(R, head_dim);
 
-  plan.v.fn<<<plan.G, plan.v.threads, plan.smem, stream>>>(tk, tv, prm);
-  cudaError_t e = cudaGetLastError();
+  // Both kernels are launched with programmatic stream serialisation: each
+  // may be scheduled while its predecessor on the stream drains, and waits
+  // for it (griddepcontrol.wait) before reading its results or writing.
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(plan.G);
+  cfg.blockDim = dim3(plan.v.threads);
+  cfg.dynamicSmemBytes = plan.smem;
+  cfg.stream = stream;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  cudaError_t e = cudaLaunchKernelEx(&cfg, plan.v.fn, tk, tv, prm);
   if (e != cudaSuccess) return fail(SF_ERR_CUDA, "verify attention launch: %s", cudaGetErrorString(e));
+  if (prm.merge_in_kernel) return SF_OK;
+  const int rpc = kMergeThreads / (head_dim / 4);
+  cfg.gridDim = dim3((R + rpc - 1) / rpc, B * H_kv);
+  cfg.blockDim = dim3(kMergeThreads);
+  cfg.dynamicSmemBytes = 0;
+  e = head_dim == 64 ? cudaLaunchKernelEx(&cfg, verify_merge_kernel<64>, prm)
+                     : cudaLaunchKernelEx(&cfg, verify_merge_kernel<128>, prm);
+  if (e != cudaSuccess) return fail(SF_ERR_CUDA, "verify merge launch: %s", cudaGetErrorString(e));
   return SF_OK;
 }
 
@@ -834,8 +1001,9 @@ extern "C" int sf_verify_attention_noalloc(const void *q, const void *k_cache,
   void *scratch = nullptr;
   st = static_scratch_address(&scratch);
   if (st != SF_OK) return st;
-  // The status word and the merge tickets must start at zero; the partials
-  // need no clearing.  The scratch keeps whatever the previous call left.
+  // The status word and the merge tickets must start at zero; descriptors
+  // and partials are written before they are read.  The scratch keeps
+  // whatever the previous call left.
   cudaError_t e = cudaMemsetAsync(scratch, 0, lay.partials_off, stream);
   if (e != cudaSuccess) return fail(SF_ERR_CUDA, "clearing the scratch: %s", cudaGetErrorString(e));
   return sf_verify_attention(q, k_cache, v_cache, block_table, seq_lens, B, n_q, H_q, H_kv,
