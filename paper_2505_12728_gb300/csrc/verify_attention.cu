@@ -59,6 +59,7 @@ struct AttnParams {
   int2 *seg_desc;     // [B * H_kv]: {first CTA, pieces} of each segment
   uint32_t *tickets;  // [B * H_kv], zero between calls (in-kernel merge)
   int merge_in_kernel;  // 1: last CTA of a segment merges; 0: merge kernel
+  int cs;             // CTAs per cluster of the launch (1: no clusters)
   float *partials;    // [G + B * H_kv][R][D + 2]
   int B, n_q, H_q, H_kv, group, R;
   int num_pages, max_pages, max_tokens;
@@ -144,6 +145,7 @@ __device__ __forceinline__ int owner_cta(long long t, long long Tot, int G) {
 }
 
 constexpr int kMergeBatch = 16;
+constexpr int kMaxCluster = 16;  // largest cluster launched (non-portable size)
 
 template <bool kBypassL1, typename T>
 __device__ __forceinline__ T merge_load(const T *p) {
@@ -249,6 +251,23 @@ verify_attention_kernel(const __grid_constant__ CUtensorMap tmap_k,
   const long long t_begin = (long long)blockIdx.x * Tot / G;
   const long long t_end = (long long)(blockIdx.x + 1) * Tot / G;
 
+  // Cluster mode: when the launch uses clusters of cs CTAs and a cluster's
+  // tiles are exactly one segment (uniform segments with G = segments x cs),
+  // its CTAs keep their partials in shared memory and combine them through
+  // distributed shared memory between two cluster barriers; no partial goes
+  // through global memory.  Decided per cluster (identically by its CTAs);
+  // every CTA of an aligned cluster has exactly one piece.
+  bool aligned = false;
+  if (p.cs > 1 && G == p.G) {
+    const long long k = blockIdx.x / p.cs;
+    const long long c0 = k * p.cs * Tot / G, c1 = (k + 1) * p.cs * Tot / G;
+    const int bb = find_sequence(c0, s_prefix, p.B, p.H_kv);
+    const int tb = s_prefix[bb + 1] - s_prefix[bb];
+    const long long base = (long long)p.H_kv * s_prefix[bb];
+    aligned = ((c0 - base) % tb == 0) && (c1 - c0 == tb);
+  }
+  int seg_b = 0, seg_h = 0;  // the segment of an aligned cluster
+
   const uint64_t policy = l2_policy_evict_first();
   bool waited = false;    // grid_dependency_wait() done
   uint32_t consumed = 0;  // tiles consumed by this CTA so far (ring position)
@@ -317,7 +336,9 @@ verify_attention_kernel(const __grid_constant__ CUtensorMap tmap_k,
       grid_dependency_wait();
       waited = true;
     }
-    if (lt0 == 0 && tid == 0) p.seg_desc[seg] = make_int2(c_first, n_pieces);
+    if (lt0 == 0 && tid == 0) p.seg_desc[seg] = make_int2(c_first, aligned ? 1 : n_pieces);
+    seg_b = b;
+    seg_h = h_kv;
 
     // ---- consumers: Q fragments of this warp's 16 rows ----
     // row r = i * g + j  <->  (draft row i, query head h_kv * g + j)
@@ -484,6 +505,10 @@ verify_attention_kernel(const __grid_constant__ CUtensorMap tmap_k,
           (void)mbar_wait_bounded(bar0 + 8 * (x % STAGES), (x / STAGES) & 1u);
       }
       __syncthreads();
+      if (aligned) {  // the cluster's other CTAs expect two barrier arrivals
+        cluster_sync();
+        cluster_sync();
+      }
       return;
     }
 
@@ -577,6 +602,33 @@ verify_attention_kernel(const __grid_constant__ CUtensorMap tmap_k,
       continue;
     }
 
+    if (aligned) {
+      // partial of this CTA's piece into its own shared memory (ring, idle):
+      // O [R][D] fp32, then m [R], l [R]; read by the cluster after the barrier
+      float *part = reinterpret_cast<float *>(smem);
+      if (writer) {
+        if (r0 < p.R) {
+#pragma unroll
+          for (int dt = 0; dt < DT; ++dt)
+            *reinterpret_cast<float2 *>(part + r0 * D + dt * 8 + colb) = make_float2(o[dt][0], o[dt][1]);
+          if ((lane & 3) == 0) {
+            part[p.R * D + r0] = m0;
+            part[p.R * D + p.R + r0] = l0;
+          }
+        }
+        if (r1 < p.R) {
+#pragma unroll
+          for (int dt = 0; dt < DT; ++dt)
+            *reinterpret_cast<float2 *>(part + r1 * D + dt * 8 + colb) = make_float2(o[dt][2], o[dt][3]);
+          if ((lane & 3) == 0) {
+            part[p.R * D + r1] = m1;
+            part[p.R * D + p.R + r1] = l1;
+          }
+        }
+      }
+      continue;
+    }
+
     // ---- several pieces: write this piece's partial ----
     const size_t stride = (size_t)p.slot_stride;
     {
@@ -632,6 +684,54 @@ verify_attention_kernel(const __grid_constant__ CUtensorMap tmap_k,
       if (tid == 0) p.tickets[seg] = 0u;
     }
     __syncthreads();
+  }
+  if (aligned) {
+    // Every CTA's partial is in its shared memory; CTA `rank` of the cluster
+    // merges rows [rank*R/cs, (rank+1)*R/cs) over the cluster's pieces, which
+    // are in rank order (= tile order), reading them through distributed
+    // shared memory.  The second barrier keeps each CTA's shared memory alive
+    // until its peers have read it.
+    cluster_sync();
+    const int cs = p.cs, rank = static_cast<int>(blockIdx.x) % cs;
+    const int R = p.R;
+    const int r_lo = rank * R / cs, r_hi = (rank + 1) * R / cs;
+    for (int idx = tid; idx < (r_hi - r_lo) * (D / 4); idx += NTHREADS) {
+      const int r = r_lo + idx / (D / 4), c4 = idx % (D / 4);
+      float mv[kMaxCluster], lv[kMaxCluster];
+      float4 xv[kMaxCluster];
+#pragma unroll
+      for (int u = 0; u < kMaxCluster; ++u) {
+        if (u < cs) {
+          mv[u] = ld_dsmem_f32(ring + 4u * (R * D + r), u);
+          lv[u] = ld_dsmem_f32(ring + 4u * (R * D + R + r), u);
+          xv[u] = ld_dsmem_f32x4(ring + 4u * (r * D + 4 * c4), u);
+        } else {
+          mv[u] = -INFINITY;
+          lv[u] = 0.f;
+          xv[u] = make_float4(0.f, 0.f, 0.f, 0.f);
+        }
+      }
+      float M = -INFINITY;
+#pragma unroll
+      for (int u = 0; u < kMaxCluster; ++u) M = fmaxf(M, mv[u]);
+      float Ls = 0.f;
+      float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+      for (int u = 0; u < kMaxCluster; ++u) {
+        const float w = exp2f(mv[u] - M);
+        Ls += lv[u] * w;
+        acc.x += xv[u].x * w; acc.y += xv[u].y * w; acc.z += xv[u].z * w; acc.w += xv[u].w * w;
+      }
+      const float inv = 1.f / Ls;
+      const int i = r / p.group, j = r % p.group;
+      const size_t row = ((size_t)seg_b * p.n_q + i) * p.H_q + (size_t)seg_h * p.group + j;
+      uint2 packed;
+      packed.x = pack_bf16x2(acc.x * inv, acc.y * inv);
+      packed.y = pack_bf16x2(acc.z * inv, acc.w * inv);
+      *reinterpret_cast<uint2 *>(p.out + row * D + 4 * c4) = packed;
+      if (p.lse && c4 == 0) p.lse[row] = (M + log2f(Ls)) * kLn2;
+    }
+    cluster_sync();
   }
 }
 
@@ -750,6 +850,7 @@ struct AttnPlan {
   AttnVariant v;
   int G;
   int smem;
+  int cs;  // CTAs per cluster (1: no clusters)
 };
 
 // Per-device, per-kernel launch facts, computed once: the dynamic shared
@@ -778,6 +879,46 @@ static int kernel_setup(const AttnVariant &v, int dev, int smem, int *occ_out) {
   return SF_OK;
 }
 
+// How many clusters of `cs` CTAs can be resident at once (cached).
+static int max_active_clusters(const AttnVariant &v, int dev, int smem, int cs, int *out) {
+  static std::mutex mu;
+  static std::map<std::tuple<void *, int, int, int>, int> cache;
+  std::lock_guard<std::mutex> lock(mu);
+  void *key = reinterpret_cast<void *>(v.fn);
+  auto it = cache.find({key, dev, smem, cs});
+  if (it == cache.end()) {
+    if (cs > 8) {
+      cudaError_t e = cudaFuncSetAttribute(v.fn, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+      if (e != cudaSuccess) {
+        cudaGetLastError();
+        it = cache.emplace(std::make_tuple(key, dev, smem, cs), 0).first;
+        *out = 0;
+        return SF_OK;
+      }
+    }
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = cs;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(cs);
+    cfg.blockDim = dim3(v.threads);
+    cfg.dynamicSmemBytes = smem;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    int n = 0;
+    cudaError_t e = cudaOccupancyMaxActiveClusters(&n, v.fn, &cfg);
+    if (e != cudaSuccess) {
+      cudaGetLastError();  // a size the device cannot run: not used
+      n = 0;
+    }
+    it = cache.emplace(std::make_tuple(key, dev, smem, cs), n).first;
+  }
+  *out = it->second;
+  return SF_OK;
+}
+
 static int plan_attention(int B, int n_q, int H_q, int H_kv, int D, int max_pages_per_seq,
                           int num_splits, AttnPlan *plan) {
   DeviceInfo dev;
@@ -794,7 +935,29 @@ static int plan_attention(int B, int n_q, int H_q, int H_kv, int D, int max_page
   if (st != SF_OK) return st;
   const long long max_tiles =
       (long long)B * H_kv * (((long long)max_pages_per_seq * SF_PAGE_SIZE + kTileTokens - 1) / kTileTokens);
-  long long G = num_splits > 0 ? num_splits : (long long)dev.sm_count * occ;
+  const long long capacity = (long long)dev.sm_count * occ;
+  long long G = num_splits > 0 ? num_splits : capacity;
+  plan->cs = 1;
+  if (num_splits <= 0 && B == 1) {
+    // One sequence: its H_kv segments have equal length, so one cluster per
+    // segment (as large as the resident capacity allows) merges on chip
+    // (cluster mode) -- provided the grid still fills most of the GPU.
+    // Batches keep the balanced global partition: their segment lengths are
+    // unknown on the host, and misaligned clusters would only cost CTAs.
+    const long long S = (long long)B * H_kv;
+    for (int cand : {8, 4, 2}) {
+      if (S * cand > capacity || S * cand > max_tiles) continue;
+      if (4 * S * cand < 3 * capacity) break;
+      int fits = 0;
+      st = max_active_clusters(plan->v, dev.ordinal, plan->smem, cand, &fits);
+      if (st != SF_OK) return st;
+      if (fits >= S) {
+        plan->cs = cand;
+        G = S * cand;
+        break;
+      }
+    }
+  }
   if (G > max_tiles) G = max_tiles;
   if (G > (1 << 20)) G = 1 << 20;
   plan->G = static_cast<int>(G < 1 ? 1 : G);
@@ -890,6 +1053,7 @@ int sf_verify_attention(const void *q, const void *k_cache, const void *v_cache,
   // of a segment merges them without a second launch.  More rows (GQA): a
   // grid-wide merge kernel spreads the larger partials over many SMs.
   prm.merge_in_kernel = R <= 16 ? 1 : 0;
+  prm.cs = plan.cs;
   prm.partials = reinterpret_cast<float *>(ws + lay.partials_off);
   prm.B = B;
   prm.n_q = n_q;
@@ -909,16 +1073,20 @@ int sf_verify_attention(const void *q, const void *k_cache, const void *v_cache,
   // Both kernels are launched with programmatic stream serialisation: each
   // may be scheduled while its predecessor on the stream drains, and waits
   // for it (griddepcontrol.wait) before reading its results or writing.
-  cudaLaunchAttribute attr[1];
+  cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
   attr[0].val.programmaticStreamSerializationAllowed = 1;
+  attr[1].id = cudaLaunchAttributeClusterDimension;
+  attr[1].val.clusterDim.x = plan.cs;
+  attr[1].val.clusterDim.y = 1;
+  attr[1].val.clusterDim.z = 1;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(plan.G);
   cfg.blockDim = dim3(plan.v.threads);
   cfg.dynamicSmemBytes = plan.smem;
   cfg.stream = stream;
   cfg.attrs = attr;
-  cfg.numAttrs = 1;
+  cfg.numAttrs = plan.cs > 1 ? 2 : 1;
   cudaError_t e = cudaLaunchKernelEx(&cfg, plan.v.fn, tk, tv, prm);
   if (e != cudaSuccess) return fail(SF_ERR_CUDA, "verify attention launch: %s", cudaGetErrorString(e));
   if (prm.merge_in_kernel) return SF_OK;
@@ -926,6 +1094,7 @@ int sf_verify_attention(const void *q, const void *k_cache, const void *v_cache,
   cfg.gridDim = dim3((R + rpc - 1) / rpc, B * H_kv);
   cfg.blockDim = dim3(kMergeThreads);
   cfg.dynamicSmemBytes = 0;
+  cfg.numAttrs = 1;  // programmatic serialisation only, no clusters
   e = head_dim == 64 ? cudaLaunchKernelEx(&cfg, verify_merge_kernel<64>, prm)
                      : cudaLaunchKernelEx(&cfg, verify_merge_kernel<128>, prm);
   if (e != cudaSuccess) return fail(SF_ERR_CUDA, "verify merge launch: %s", cudaGetErrorString(e));

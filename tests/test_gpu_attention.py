@@ -178,3 +178,22 @@ def test_invalid_arguments_raise_before_launch():
     with pytest.raises(sfv.SFError):      # workspace too small
         sfv.verify_attention(dev["q"], dev["k_cache"], dev["v_cache"], dev["block_table"],
                              dev["seq_lens"], workspace=sfv.new_workspace(256))
+
+
+@pytest.mark.parametrize("B,n_q,H_q,H_kv,d,prefix", [
+    (1, 5, 32, 32, 128, 3008),     # one sequence, MHA: one 8-CTA cluster per KV head
+    (1, 8, 128, 32, 128, 2000),    # one sequence, 32 rows per KV head
+    (1, 7, 224, 32, 64, 700),      # one sequence, 49 rows per KV head, d = 64
+    (2, 8, 28, 4, 128, 2000),      # equal-length batch (balanced global partition)
+])
+def test_uniform_segments_match_oracle(oracle_mod, B, n_q, H_q, H_kv, d, prefix):
+    # With the automatic split count a single sequence's segments are each
+    # covered by one thread-block cluster whose CTAs merge through
+    # distributed shared memory; results must match the oracle like every
+    # other path, and repeat bit for bit.
+    case = make_attention_case(B, n_q, H_q, H_kv, d, [prefix] * B, seed=900 + B + n_q)
+    ref_out, ref_lse = oracle_attention(oracle_mod, case)
+    out, lse = run_attention(case, num_splits=0)
+    assert_attention_close(out, lse, ref_out, ref_lse)
+    out2, lse2 = run_attention(case, num_splits=0)
+    np.testing.assert_array_equal(out, out2)
