@@ -11,7 +11,10 @@ streams the caches from HBM.
 Prints ONE JSON line (rank 0).  `value` is draft tokens verified per second
 over the whole job; `e2e` repeats the measurement through host buffers
 (pinned host -> device copies of the step's inputs and a device -> host read
-of its results inside the timed region).
+of its results inside the timed region).  The step is captured once into
+CUDA graphs (the C-ABI calls are asynchronous and allocation-free) and
+replayed, as a serving loop would; `--eager` launches every call from Python
+instead (then the host, not the GPU, sets the pace).
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME]
   python bench.py --impl reference ...   # the CPU oracle, same metric
@@ -288,7 +291,9 @@ def run_ours(args):
     ws_att = sfv.new_workspace(sfv.verify_attention_workspace_size(
         wl.B, wl.rows, wl.H_q, wl.H_kv, wl.d, att.block_table.shape[2]), dev)
     ws_acc = sfv.new_workspace(sfv.accept_workspace_size(wl.B, wl.k, wl.V), dev)
-    stream = torch.cuda.current_stream()
+    torch.cuda.synchronize()
+    stream = torch.cuda.Stream()          # a non-default stream (graphs are captured on it)
+    torch.cuda.set_stream(stream)
 
     def attention_layers(qsrc):
         for l in range(L):
@@ -307,10 +312,41 @@ def run_ours(args):
         step()
     torch.cuda.synchronize()
 
-    # ---- device-resident timing ----
-    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(args.steps)]
+    # ---- eager timing (Python launches every call; host-bound, for reference) ----
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(args.steps):
+        step()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    eager_ms = e0.elapsed_time(e1) / args.steps
+
+    # ---- the step as CUDA graphs: all attention layers, then the acceptance ----
+    def capture(fn):
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=stream):
+            fn()
+        return g
+
+    use_graph = not args.eager
+    if use_graph:
+        g_att = capture(lambda: attention_layers(q))
+        g_acc = capture(lambda: acceptance(logits, qprob, toks, uni, temp))
+        run_att, run_acc = g_att.replay, g_acc.replay
+    else:
+        run_att = lambda: attention_layers(q)
+        run_acc = lambda: acceptance(logits, qprob, toks, uni, temp)
+    # clocks are sampled from the warm-up through the end of the timed region
     clocks = ClockSampler(local)
     clocks.start()
+    for _ in range(args.warmup):
+        run_att()
+        run_acc()
+    torch.cuda.synchronize()
+
+    # ---- device-resident timing ----
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(args.steps)]
     barrier(world)
     torch.cuda.synchronize()
     t_start = torch.cuda.Event(enable_timing=True)
@@ -318,9 +354,9 @@ def run_ours(args):
     t_start.record(stream)
     for s in range(args.steps):
         ev[s][0].record(stream)
-        attention_layers(q)
+        run_att()
         ev[s][1].record(stream)
-        acceptance(logits, qprob, toks, uni, temp)
+        run_acc()
         ev[s][2].record(stream)
     t_end.record(stream)
     torch.cuda.synchronize()
@@ -361,17 +397,20 @@ def run_ours(args):
     for _ in range(args.warmup):
         e2e_step()
     torch.cuda.synchronize()
+    run_e2e = capture(e2e_step).replay if use_graph else e2e_step
+    for _ in range(args.warmup):
+        run_e2e()
+    torch.cuda.synchronize()
     barrier(world)
-    e0 = torch.cuda.Event(enable_timing=True)
-    e1 = torch.cuda.Event(enable_timing=True)
     e0.record(stream)
     for _ in range(args.steps):
-        e2e_step()
+        run_e2e()
     e1.record(stream)
     torch.cuda.synchronize()
     barrier(world)
     e2e_ms = max_over_ranks(e0.elapsed_time(e1), world, dev)
     e2e_value = tokens / (e2e_ms / 1e3)
+    h_ok = bool(np.array_equal(h_n.numpy(), n_acc.cpu().numpy()))
 
     # ---- roofline of the dominant kernel (verification attention) ----
     peak, peak_kind = measured_peaks()
@@ -399,8 +438,11 @@ def run_ours(args):
                      "kernel": "verify_attention_kernel",
                      "peak_source": f"{peak_kind} copy bandwidth (MEASURED_PEAKS.json hbm_gbs)"},
         "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d,
-                "d2h_bytes_per_step": d2h, "ms_per_step": e2e_ms / args.steps},
-        "gpu_launches": args.steps * (L + 2),
+                "d2h_bytes_per_step": d2h, "ms_per_step": e2e_ms / args.steps,
+                "host_result_matches_device": h_ok},
+        "launch": "cuda_graph" if use_graph else "eager",
+        "eager_ms_per_step": eager_ms,
+        "gpu_launches": args.steps * (L * (1 if wl.rows <= 16 else 2) + 2),
         "clocks": clk,
         "device_status": status,
     }
@@ -416,13 +458,15 @@ def run_ours(args):
 def main(argv=None):
     ap = argparse.ArgumentParser(description=__doc__.split("\n")[0])
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=20)
-    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--steps", type=int, default=400)
+    ap.add_argument("--warmup", type=int, default=50)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", default="image7b")
     ap.add_argument("--cpu-budget", type=float, default=12.0,
                     help="seconds of oracle work for the cpu_baseline sample")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--eager", action="store_true",
+                    help="launch every call from Python instead of replaying CUDA graphs")
     args = ap.parse_args(argv)
     args.warmup = max(3, args.warmup)   # at least 3 untimed warm-up steps
     if args.impl == "reference":
