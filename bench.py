@@ -145,6 +145,34 @@ def accept_bytes(wl, mode_sampling_rows: int) -> int:
     return wl.B * (wl.k + 1) * wl.V * 4 + mode_sampling_rows * wl.V * 4 * 2
 
 
+def profiled_traffic(kernel_sources, profile):
+    """DRAM bytes per launch from a committed ncu summary, or None when the
+    kernel's sources changed since the counters were taken."""
+    import hashlib
+    import re
+    try:
+        h = hashlib.sha256()
+        for f in kernel_sources:
+            with open(os.path.join(ROOT, f)) as fh:
+                code = fh.read()
+            # the code only: comments and layout do not change the kernel
+            code = re.sub(r"/\*.*?\*/", "", code, flags=re.S)
+            code = re.sub(r"//[^\n]*", "", code)
+            h.update("".join(code.split()).encode())
+        with open(os.path.join(ROOT, profile)) as fh:
+            text = fh.read()
+    except OSError:
+        return None
+    fields = dict(line.split(":", 1) for line in text.splitlines()
+                  if line.startswith(("kernel_source_sha256_16:", "traffic_bytes_per_launch:")))
+    if fields.get("kernel_source_sha256_16", "").strip() != h.hexdigest()[:16]:
+        return None
+    try:
+        return int(fields["traffic_bytes_per_launch"])
+    except (KeyError, ValueError):
+        return None
+
+
 def measured_peaks():
     try:
         with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
@@ -434,7 +462,13 @@ def run_ours(args):
         "accept_gbs": accept_bytes(wl, sampling_rows) / (acc_launch_ms / 1e3) / 1e9,
         "mean_accepted": float(n_acc.float().mean().item()),
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
-                     "frac": achieved / peak, "traffic": None,
+                     "frac": achieved / peak,
+                     "traffic": (profiled_traffic(
+                         ["paper_2505_12728_gb300/csrc/verify_attention.cu",
+                          "paper_2505_12728_gb300/csrc/sf_device.cuh"],
+                         "profiles/verify_attention_image7b.md")
+                         if wl.name == "image7b" else None),
+                     "algorithmic_bytes": bytes_layer,
                      "kernel": "verify_attention_kernel",
                      "peak_source": f"{peak_kind} copy bandwidth (MEASURED_PEAKS.json hbm_gbs)"},
         "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d,

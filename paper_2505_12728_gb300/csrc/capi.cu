@@ -49,9 +49,8 @@ typedef CUresult (*EncodeTiledFn)(CUtensorMap *, CUtensorMapDataType, cuuint32_t
                                   const cuuint32_t *, CUtensorMapInterleave, CUtensorMapSwizzle,
                                   CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
 
-int encode_tensor_map_2d_bf16(CUtensorMap *map, const void *base, uint64_t inner_elems,
-                              uint64_t rows, uint64_t row_stride_bytes, uint32_t box_inner,
-                              uint32_t box_rows, bool swizzle_128b) {
+int encode_tensor_map_bf16(CUtensorMap *map, const void *base, int rank, const uint64_t *dims,
+                           const uint64_t *strides, const uint32_t *box) {
   static std::once_flag once;
   static EncodeTiledFn fn = nullptr;
   static cudaError_t fetch_err = cudaSuccess;
@@ -66,13 +65,17 @@ int encode_tensor_map_2d_bf16(CUtensorMap *map, const void *base, uint64_t inner
   if (!fn)
     return fail(SF_ERR_CUDA, "cuTensorMapEncodeTiled unavailable (%s)",
                 cudaGetErrorString(fetch_err));
-  cuuint64_t dims[2] = {inner_elems, rows};
-  cuuint64_t strides[1] = {row_stride_bytes};
-  cuuint32_t box[2] = {box_inner, box_rows};
-  cuuint32_t estr[2] = {1, 1};
-  CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(base), dims,
-                  strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
-                  swizzle_128b ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_NONE,
+  if (rank < 1 || rank > 5) return fail(SF_ERR_INVALID_ARG, "tensor map rank %d", rank);
+  cuuint64_t d[5], st[4];
+  cuuint32_t bx[5], es[5];
+  for (int i = 0; i < rank; ++i) {
+    d[i] = dims[i];
+    bx[i] = box[i];
+    es[i] = 1;
+    if (i + 1 < rank) st[i] = strides[i];
+  }
+  CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, rank, const_cast<void *>(base), d, st, bx,
+                  es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
                   CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   if (r != CUDA_SUCCESS) return fail(SF_ERR_CUDA, "cuTensorMapEncodeTiled failed (CUresult %d)", (int)r);
   return SF_OK;

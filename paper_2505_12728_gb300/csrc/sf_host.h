@@ -25,10 +25,11 @@ struct DeviceInfo {
 };
 int current_device(DeviceInfo *info);
 
-// cuTensorMapEncodeTiled fetched through the runtime (no link-time libcuda).
-int encode_tensor_map_2d_bf16(CUtensorMap *map, const void *base, uint64_t inner_elems,
-                              uint64_t rows, uint64_t row_stride_bytes, uint32_t box_inner,
-                              uint32_t box_rows, bool swizzle_128b);
+// cuTensorMapEncodeTiled for a bf16 tensor of `rank` dimensions (dims[0]
+// innermost; strides[i] is the byte stride of dimension i+1), fetched
+// through the runtime (no link-time libcuda).  128-byte swizzle, zero fill.
+int encode_tensor_map_bf16(CUtensorMap *map, const void *base, int rank, const uint64_t *dims,
+                           const uint64_t *strides, const uint32_t *box);
 
 inline bool aligned(const void *p, size_t a) {
   return (reinterpret_cast<uintptr_t>(p) % a) == 0;

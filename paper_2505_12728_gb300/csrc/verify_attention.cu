@@ -10,25 +10,31 @@
 // GB300 design (the paper gives no kernel; its runs used one A6000):
 //  * Work unit = a tile of 64 cached tokens of one (sequence, KV head)
 //    "segment".  All tiles of the batch form one ordered list that is cut
-//    into G equal, contiguous ranges, one per CTA (G = SMs x resident CTAs),
-//    so long and short sequences balance without any host-side knowledge of
-//    seq_lens.  A CTA's range touches one or two segments ("pieces").
+//    into G equal, contiguous ranges, one per CTA, computed on the device from
+//    seq_lens, so long and short sequences balance without host knowledge of
+//    the lengths.  A CTA's range touches one or two segments ("pieces").
 //  * Each CTA streams its tiles through a STAGES-deep ring in shared memory:
-//    one elected warp issues 2-D TMA copies of whole 16-token pages (128-byte
-//    swizzled boxes, one per page, half head_dim and tensor) straight from
-//    the block table into the ring, completing on an mbarrier; nothing else
-//    touches HBM in the loop.
+//    one elected warp issues one TMA box per 16-token page and tensor
+//    (128-byte swizzle) straight from the block table, completing on an
+//    mbarrier; nothing else touches HBM in the loop.
 //  * All n_q * g query rows of a KV head share each K/V tile.  The rows are
 //    the M dimension of bf16 m16n8k16 tensor-core MMAs (S = Q K^T and
 //    O += P V, fp32 accumulate); scores stay in registers, where an fp32
-//    online softmax (base-2, scale folded in) rescales the running output.
+//    online softmax (base 2, scale folded in) rescales the running output.
 //    With one row tile (MHA, n_q <= 16) the four warps split the tile's keys
 //    and combine in shared memory at the end of a piece.
 //  * A piece that covers a whole segment writes bf16 out and fp32 LSE
-//    directly.  Otherwise it writes an fp32 partial (O unnormalised, running
-//    max, running sum) to the workspace, and the CTA that takes the last
-//    ticket of the segment (an atomic counter; nobody waits) merges all
-//    partials in piece order, so results are deterministic.
+//    directly.  Split segments are merged (deterministically, in piece
+//    order) in one of three ways:
+//      - cluster mode: for one sequence the grid is one thread-block cluster
+//        per KV head; the cluster's CTAs keep their partials in shared
+//        memory and merge them through distributed shared memory;
+//      - few rows (R <= 16): the CTA that takes the last ticket of the
+//        segment (an atomic counter; nobody waits) merges the fp32 partials;
+//      - many rows (GQA): verify_merge_kernel, a grid over rows and segments.
+//  * Launches use programmatic stream serialisation: the partition, the
+//    block-table reads and the first copies run before griddepcontrol.wait,
+//    overlapping the previous kernel on the stream.
 //  * Page indices outside the pool and positions past a sequence's end are
 //    loaded as zero boxes (TMA out-of-bounds fill); bad indices set a bit in
 //    the status word.  Every mbarrier wait is bounded.
@@ -46,7 +52,6 @@ constexpr int kTileTokens = 64;            // keys per ring stage
 constexpr int kPageTokens = SF_PAGE_SIZE;  // 16
 constexpr int kPagesPerTile = kTileTokens / kPageTokens;
 constexpr int kRowBytes = 128;             // one swizzled smem row (64 bf16)
-constexpr int kHalfBytes = kTileTokens * kRowBytes;  // 64 tokens x 128 B
 constexpr int kBeyondEnd = -2147483647 - 1;           // page past the sequence end
 
 struct AttnParams {
@@ -74,11 +79,14 @@ __host__ __device__ inline int partial_slot_floats(int R, int D) {
   return (R * (D + 2) + 3) / 4 * 4;
 }
 
-// Byte offset of 16-byte chunk `c` (head_dim / 8 index) of token `t` inside a
-// tile written by 128B-swizzled TMA boxes: [c / 8][t][(c % 8) ^ (t % 8)].
+// Shared-memory layout of one K or V tile (64 tokens): one TMA box per page,
+// [page][c / 8][token % 16][128 B], each 128-byte row 128B-swizzled.  Byte
+// offset of 16-byte chunk `c` (head_dim / 8 index) of token `t`:
+template <int D>
 __device__ __forceinline__ uint32_t swz(int t, int c) {
-  return static_cast<uint32_t>((c >> 3) * kHalfBytes + t * kRowBytes +
-                               (((c & 7) ^ (t & 7)) << 4));
+  constexpr int kPageBytes = (D / 64) * kPageTokens * kRowBytes;
+  return static_cast<uint32_t>((t >> 4) * kPageBytes + (c >> 3) * (kPageTokens * kRowBytes) +
+                               (t & 15) * kRowBytes + (((c & 7) ^ (t & 7)) << 4));
 }
 
 template <int D, int STAGES, int NW>
@@ -307,13 +315,15 @@ verify_attention_kernel(const __grid_constant__ CUtensorMap tmap_k,
         if (phys < 0 || phys >= p.num_pages) set_status(p.status, SF_DEVICE_BAD_PAGE);
         else row = (phys * p.H_kv + h_kv) * kPageTokens;
       }
-      const uint32_t dst = ring + slot * L::kStageBytes + pg * kPageTokens * kRowBytes;
+      const uint32_t dst = ring + slot * L::kStageBytes + pg * HALVES * kPageTokens * kRowBytes;
       const uint32_t bar = bar0 + 8 * slot;
-#pragma unroll
-      for (int hf = 0; hf < HALVES; ++hf) {
-        tma_load_2d(dst + hf * kHalfBytes, &tmap_k, hf * 64, row, bar, policy);
-        tma_load_2d(dst + L::kTensorTileBytes + hf * kHalfBytes, &tmap_v, hf * 64, row, bar,
-                    policy);
+      if constexpr (HALVES == 2) {
+        // both 128-byte column halves of the page in one box (3-D map)
+        tma_load_3d(dst, &tmap_k, 0, row, 0, bar, policy);
+        tma_load_3d(dst + L::kTensorTileBytes, &tmap_v, 0, row, 0, bar, policy);
+      } else {
+        tma_load_2d(dst, &tmap_k, 0, row, bar, policy);
+        tma_load_2d(dst + L::kTensorTileBytes, &tmap_v, 0, row, bar, policy);
       }
     };
 
@@ -389,8 +399,10 @@ verify_attention_kernel(const __grid_constant__ CUtensorMap tmap_k,
           for (int idx = tid; idx < (kTileTokens - valid) * HALVES * 8; idx += NTHREADS) {
             const int tok = valid + idx / (HALVES * 8);
             const int rem = idx % (HALVES * 8);
-            *reinterpret_cast<uint4 *>(vt + (rem >> 3) * kHalfBytes + tok * kRowBytes +
-                                       (rem & 7) * 16) = make_uint4(0, 0, 0, 0);
+            *reinterpret_cast<uint4 *>(vt + (tok >> 4) * (HALVES * kPageTokens * kRowBytes) +
+                                       (rem >> 3) * (kPageTokens * kRowBytes) +
+                                       (tok & 15) * kRowBytes + (rem & 7) * 16) =
+                make_uint4(0, 0, 0, 0);
           }
           fence_proxy_async_smem();
         }
@@ -408,7 +420,7 @@ verify_attention_kernel(const __grid_constant__ CUtensorMap tmap_k,
           for (int nt = 0; nt < NT; ++nt) {
             const int key = ks * KW + nt * 8 + (lane & 7);
             uint32_t b0, b1, b2, b3;
-            ldmatrix_x4(kbase + swz(key, 2 * kk + (lane >> 3)), b0, b1, b2, b3);
+            ldmatrix_x4(kbase + swz<D>(key, 2 * kk + (lane >> 3)), b0, b1, b2, b3);
             mma_bf16_16816(s[nt], qa[kk], b0, b1);
             mma_bf16_16816(s[nt], qa[kk + 1], b2, b3);
           }
@@ -473,7 +485,7 @@ verify_attention_kernel(const __grid_constant__ CUtensorMap tmap_k,
 #pragma unroll
           for (int dt = 0; dt < DT; dt += 2) {
             uint32_t b0, b1, b2, b3;
-            ldmatrix_x4_trans(vbase + swz(key, dt + (lane >> 4)), b0, b1, b2, b3);
+            ldmatrix_x4_trans(vbase + swz<D>(key, dt + (lane >> 4)), b0, b1, b2, b3);
             mma_bf16_16816(o[dt], pa, b0, b1);
             mma_bf16_16816(o[dt + 1], pa, b2, b3);
           }
@@ -977,8 +989,20 @@ static int cache_tensor_map(CUtensorMap *out, const void *base, uint64_t rows, i
       return SF_OK;
     }
   }
-  int st = encode_tensor_map_2d_bf16(out, base, head_dim, rows, (uint64_t)head_dim * 2, 64,
-                                     SF_PAGE_SIZE, true);
+  // head_dim 128: view each 256-byte token row as two 128-byte halves with
+  // the halves outermost, {64 elements, rows, 2 halves} with byte strides
+  // {256, 128}, so a {64, 16, 2} box brings a whole page in the shared
+  // layout [half][token][64].  head_dim 64: {64, rows}, box {64, 16}.
+  int st;
+  if (head_dim == 128) {
+    const uint64_t dims[3] = {64, rows, 2}, strides[2] = {256, 128};
+    const uint32_t box[3] = {64, SF_PAGE_SIZE, 2};
+    st = encode_tensor_map_bf16(out, base, 3, dims, strides, box);
+  } else {
+    const uint64_t dims[2] = {64, rows}, strides[1] = {128};
+    const uint32_t box[2] = {64, SF_PAGE_SIZE};
+    st = encode_tensor_map_bf16(out, base, 2, dims, strides, box);
+  }
   if (st != SF_OK) return st;
   std::lock_guard<std::mutex> lock(mu);
   if (maps.size() >= 4096) maps.clear();
