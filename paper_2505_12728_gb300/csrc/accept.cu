@@ -11,19 +11,28 @@
 //
 // GB300 design.  The whole cost is streaming the (k+1) x V fp32 logits once
 // (plus one row of q for the draw), so both kernels are coalesced 128-bit
-// streaming reductions spread over many CTAs, with no tensor cores:
+// streaming reductions spread over many CTAs, with no tensor cores, and the
+// critical path is a short chain of memory round trips:
 //  * accept_stats_kernel, grid (chunks, k+1, B): each CTA reduces a chunk of
-//    one row to (max, first argmax, sum exp((x - max)/tau)) with the chunk
-//    held in registers; the last CTA of a row (atomic ticket, nobody waits)
-//    combines the chunks in fp64; the last row of a sequence to finish takes
-//    the k accept/reject decisions in fp64 and writes the accepted tokens.
-//  * accept_draw_kernel, grid (chunks, B): for sampled sequences, each CTA
-//    sums the residual (or bonus) mass of a chunk of row j; the last CTA of
-//    the sequence locates the chunk holding u_k * S with an fp64 scan over
-//    the chunk sums, then scans that chunk element by element in ascending
+//    one row to (max, first argmax, sum exp((x - max)/tau)) with the chunk in
+//    registers; the CTA whose chunk holds the row's draft token also records
+//    that token's logit and draft probability.  The last CTA of a sequence
+//    to finish (one atomic ticket; nobody waits) combines every row, one warp
+//    per row, in fp64, and takes the k accept/reject decisions in fp64.
+//  * accept_draw_kernel, grid (chunks, B), launched with programmatic stream
+//    serialisation so that it is resident while the first kernel drains: for
+//    sampled sequences each CTA sums the residual (or bonus) mass of a chunk
+//    of row j; the last CTA of the sequence locates the chunk holding u_k * S
+//    with an fp64 scan over chunk sums and scans that chunk in ascending
 //    token order.
-// Per-element arithmetic is fp32 (expf, explicitly rounded products and
-// differences, identical in both passes); every sum above one thread is fp64.
+// Arithmetic: per-element terms are fp32 (expf, explicitly rounded products
+// and differences, identical wherever a value is recomputed); sums, scans and
+// the accept tests use float-float numbers (an unevaluated sum hi + lo of two
+// fp32 values, ~44 significant bits) built from exactly rounded fp32
+// operations, accumulated in a fixed order (results are deterministic).
+// GB300's fp64 pipe is far too slow for this latency-bound path, and
+// float-float gives the accuracy the decisions need.
+#include <climits>
 #include <cmath>
 
 #include "sf_device.cuh"
@@ -32,13 +41,28 @@
 namespace sf {
 
 constexpr int kAccThreads = 256;
+constexpr int kAccWarps = kAccThreads / 32;
 constexpr int kMaxPerThread = 32;                       // elements held per thread
 constexpr int kMaxChunk = kAccThreads * kMaxPerThread;  // 8192 elements per CTA
 
-struct RowStat {   // one (sequence, row) or one chunk of it
-  float m;         // largest raw logit
+struct ff {       // float-float number hi + lo, |lo| <= ulp(hi) / 2
+  float hi, lo;
+};
+
+struct ChunkRec {  // one chunk of one target row
+  float m;         // largest raw logit in the chunk
   int arg;         // its first index
-  double S;        // sum of exp((x - m) / tau); 0 for greedy rows
+  ff S;            // sum of exp((x - m) / tau) over the chunk; 0 for greedy rows
+  float lx;        // logit of the row's draft token, if it lies in this chunk
+  float qx;        // its draft probability
+  int has_x;       // 1 if the row's draft token lies in this chunk
+  int pad;
+};
+
+struct RowStat {   // one combined target row
+  float m;
+  int arg;
+  ff S;
 };
 
 struct SeqState {
@@ -47,34 +71,33 @@ struct SeqState {
 };
 
 struct DrawPart {
-  double sum_r;    // residual (or bonus) mass of the chunk
-  double sum_p;    // target mass of the chunk (fallback when the residual is 0)
+  ff sum_r;        // residual (or bonus) mass of the chunk
+  ff sum_p;        // target mass of the chunk (fallback when the residual is 0)
   int last_r;      // last index with r > 0 (-1 if none)
   int last_p;      // last index with p > 0 (-1 if none)
   int pad[2];
 };
 
 struct AccParams {
-  const float *logits;   // [B][k+1][V]
-  const float *q;        // [B][k][V]
-  const int32_t *tokens; // [B][k]
-  const float *u;        // [B][k+1]
-  const float *tau;      // [B]
-  int32_t *num_accepted; // [B]
-  int32_t *out_tokens;   // [B][k+1]
-  float *ratio;          // [B][k] or null
+  const float *logits;     // [B][k+1][V]
+  const float *q;          // [B][k][V]
+  const int32_t *tokens;   // [B][k]
+  const float *u;          // [B][k+1]
+  const float *tau;        // [B]
+  int32_t *num_accepted;   // [B]
+  int32_t *out_tokens;     // [B][k+1]
+  float *ratio;            // [B][k] or null
   uint32_t *status;
-  uint32_t *row_tickets; // [B][k+1]
-  uint32_t *seq_tickets; // [B]
-  uint32_t *draw_tickets;// [B]
-  RowStat *rows;         // [B][k+1]
-  RowStat *chunks;       // [B][k+1][C1]
-  SeqState *seqs;        // [B]
-  DrawPart *parts;       // [B][C2]
+  uint32_t *seq_tickets;   // [B]
+  uint32_t *draw_tickets;  // [B]
+  ChunkRec *chunks;        // [B][k+1][C1]
+  RowStat *rows;           // [B][k+1]
+  SeqState *seqs;          // [B]
+  DrawPart *parts;         // [B][C2]
   int B, k, V;
-  int C1, CV1;           // stats chunks per row, elements per chunk
-  int C2, CV2;           // draw chunks per row, elements per chunk
-  int vec4;              // rows are 16-byte aligned and V % 4 == 0
+  int C1, CV1;             // stats chunks per row, elements per chunk
+  int C2, CV2;             // draw chunks per row, elements per chunk
+  int vec4;                // rows are 16-byte aligned and V % 4 == 0
 };
 
 // (value, index) order for argmax: larger value first, then lower index.
@@ -94,23 +117,89 @@ __device__ __forceinline__ void draw_terms(float x, float qx, bool residual, flo
   r = residual ? fmaxf(__fsub_rn(pz, qx), 0.0f) : pz;
 }
 
-template <typename T>
-__device__ __forceinline__ T warp_sum(T v) {
+// Float-float arithmetic (Knuth's TwoSum and an FMA-based TwoProduct); the
+// explicit _rn intrinsics keep the compiler from contracting or reordering.
+__device__ __forceinline__ ff ff_of(float x) { return ff{x, 0.f}; }
+
+__device__ __forceinline__ ff ff_add(ff a, ff b) {
+  const float s = __fadd_rn(a.hi, b.hi);
+  const float v = __fsub_rn(s, a.hi);
+  float e = __fadd_rn(__fsub_rn(a.hi, __fsub_rn(s, v)), __fsub_rn(b.hi, v));
+  e = __fadd_rn(e, __fadd_rn(a.lo, b.lo));
+  const float hi = __fadd_rn(s, e);
+  return ff{hi, __fsub_rn(e, __fsub_rn(hi, s))};
+}
+
+__device__ __forceinline__ ff ff_mul(ff a, float b) {
+  const float p = __fmul_rn(a.hi, b);
+  float e = __fmaf_rn(a.hi, b, -p);
+  e = __fmaf_rn(a.lo, b, e);
+  const float hi = __fadd_rn(p, e);
+  return ff{hi, __fsub_rn(e, __fsub_rn(hi, p))};
+}
+
+__device__ __forceinline__ bool ff_lt(ff a, ff b) {
+  return a.hi < b.hi || (a.hi == b.hi && a.lo < b.lo);
+}
+
+__device__ __forceinline__ bool ff_pos(ff a) { return a.hi > 0.f || (a.hi == 0.f && a.lo > 0.f); }
+
+// a / b rounded to fp32 (one Newton correction of the fp32 quotient).
+__device__ __forceinline__ float ff_div_to_f(float a, ff b) {
+  const float q = __fdiv_rn(a, b.hi);
+  float r = __fmaf_rn(-q, b.hi, a);  // a - q * b.hi, exact
+  r = __fmaf_rn(-q, b.lo, r);
+  return __fadd_rn(q, __fdiv_rn(r, b.hi));
+}
+
+// exp((x - m) / tau) with the argument carried to float-float, so that the
+// result is as accurate as expf itself even for large |x - m|.
+__device__ __forceinline__ float exp_diff_accurate(float x, float m, float tau) {
+  float hi = __fsub_rn(x, m);
+  const float v = __fsub_rn(hi, x);
+  float lo = __fadd_rn(__fsub_rn(x, __fsub_rn(hi, v)), __fsub_rn(-m, v));
+  if (tau != 1.0f) {
+    const float qh = __fdiv_rn(hi, tau);
+    const float r = __fmaf_rn(-qh, tau, hi);  // hi - qh * tau, exact
+    lo = __fdiv_rn(__fadd_rn(r, lo), tau);
+    hi = qh;
+  }
+  return __fmul_rn(expf(hi), __fadd_rn(1.0f, lo));
+}
+
+__device__ __forceinline__ ff shfl_xor_ff(ff a, int o) {
+  return ff{__shfl_xor_sync(0xffffffffu, a.hi, o), __shfl_xor_sync(0xffffffffu, a.lo, o)};
+}
+
+__device__ __forceinline__ ff shfl_up_ff(ff a, int o) {
+  return ff{__shfl_up_sync(0xffffffffu, a.hi, o), __shfl_up_sync(0xffffffffu, a.lo, o)};
+}
+
+__device__ __forceinline__ ff warp_sum_ff(ff v) {
 #pragma unroll
-  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  for (int o = 16; o > 0; o >>= 1) v = ff_add(v, shfl_xor_ff(v, o));
   return v;
 }
 
-// Block-wide sum in fp64 (deterministic tree order).
-__device__ double block_sum(double v, double *s_buf) {
+__device__ __forceinline__ void warp_argmax(float &v, int &i) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    const float ov = __shfl_xor_sync(0xffffffffu, v, o);
+    const int oi = __shfl_xor_sync(0xffffffffu, i, o);
+    if (better(ov, oi, v, i)) { v = ov; i = oi; }
+  }
+}
+
+// Block-wide float-float sum (fixed tree order).
+__device__ ff block_sum(ff v, ff *s_buf) {
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  v = warp_sum(v);
+  v = warp_sum_ff(v);
   __syncthreads();
   if (lane == 0) s_buf[warp] = v;
   __syncthreads();
   if (warp == 0) {
-    v = lane < kAccThreads / 32 ? s_buf[lane] : 0.0;
-    v = warp_sum(v);
+    v = lane < kAccWarps ? s_buf[lane] : ff_of(0.f);
+    v = warp_sum_ff(v);
     if (lane == 0) s_buf[0] = v;
   }
   __syncthreads();
@@ -119,24 +208,14 @@ __device__ double block_sum(double v, double *s_buf) {
 
 __device__ void block_argmax(float &v, int &i, float *s_v, int *s_i) {
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) {
-    const float ov = __shfl_xor_sync(0xffffffffu, v, o);
-    const int oi = __shfl_xor_sync(0xffffffffu, i, o);
-    if (better(ov, oi, v, i)) { v = ov; i = oi; }
-  }
+  warp_argmax(v, i);
   __syncthreads();
   if (lane == 0) { s_v[warp] = v; s_i[warp] = i; }
   __syncthreads();
   if (warp == 0) {
-    v = lane < kAccThreads / 32 ? s_v[lane] : -INFINITY;
-    i = lane < kAccThreads / 32 ? s_i[lane] : 0x7fffffff;
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) {
-      const float ov = __shfl_xor_sync(0xffffffffu, v, o);
-      const int oi = __shfl_xor_sync(0xffffffffu, i, o);
-      if (better(ov, oi, v, i)) { v = ov; i = oi; }
-    }
+    v = lane < kAccWarps ? s_v[lane] : -INFINITY;
+    i = lane < kAccWarps ? s_i[lane] : INT_MAX;
+    warp_argmax(v, i);
     if (lane == 0) { s_v[0] = v; s_i[0] = i; }
   }
   __syncthreads();
@@ -144,16 +223,60 @@ __device__ void block_argmax(float &v, int &i, float *s_v, int *s_i) {
   i = s_i[0];
 }
 
+// Inclusive float-float prefix sum over the block (fixed order).  Returns
+// the thread's inclusive value; *excl receives its exclusive value (the
+// previous thread's inclusive value, bit for bit) and *total the block total
+// (the last thread's inclusive value).  s_buf holds kAccWarps + 1 values.
+__device__ ff block_inclusive_scan(ff v, ff *s_buf, ff *excl, ff *total) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const ff n = shfl_up_ff(v, o);
+    if (lane >= o) v = ff_add(n, v);
+  }
+  __syncthreads();
+  if (lane == 31) s_buf[warp] = v;  // warp totals
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    // warp offsets in sequence: off(w) = ff_add(off(w-1), t(w-1)) is, bit for
+    // bit, the inclusive value of the last thread of warp w-1
+    ff off = ff_of(0.f);
+    for (int w = 0; w < kAccWarps; ++w) {
+      const ff t = s_buf[w];
+      s_buf[w] = off;
+      off = ff_add(off, t);
+    }
+    s_buf[kAccWarps] = off;
+  }
+  __syncthreads();
+  const ff off = s_buf[warp];
+  const ff incl = ff_add(off, v);
+  const ff prev = shfl_up_ff(incl, 1);
+  *excl = lane > 0 ? prev : off;
+  *total = s_buf[kAccWarps];
+  __syncthreads();  // s_buf is reused by the next call
+  return incl;
+}
+
 __global__ void __launch_bounds__(kAccThreads)
 accept_stats_kernel(const __grid_constant__ AccParams p) {
-  __shared__ double s_d[32];
+  __shared__ ff s_d[32];
   __shared__ float s_v[32];
   __shared__ int s_i[32];
   __shared__ int s_flag;
   __shared__ int s_acc[SF_MAX_DRAFT];
+  __shared__ float s_rm[SF_MAX_DRAFT + 1], s_rlx[SF_MAX_DRAFT + 1], s_rqx[SF_MAX_DRAFT + 1];
+  __shared__ int s_rarg[SF_MAX_DRAFT + 1], s_rhx[SF_MAX_DRAFT + 1];
+  __shared__ ff s_rS[SF_MAX_DRAFT + 1];
+
+  // The next kernel (the draw) may be scheduled as CTAs of this grid finish.
+  // Inputs are read before grid_dependency_wait() (this library's kernels,
+  // the only ones that let their successor start early, never write them);
+  // the workspace and the outputs are written only after it.
+  grid_launch_dependents();
 
   const int c = blockIdx.x, r = blockIdx.y, b = blockIdx.z;
-  const int tid = threadIdx.x;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int k = p.k, V = p.V;
   const float tau = p.tau[b];
   const bool greedy = !(tau > 0.0f);
@@ -161,11 +284,20 @@ accept_stats_kernel(const __grid_constant__ AccParams p) {
   const int c0 = c * p.CV1;
   const int c1 = min(V, c0 + p.CV1);
 
+  // the row's draft token, and the decision inputs (used by the last CTA)
+  const int x_row = r < k ? p.tokens[(size_t)b * k + r] : -1;
+  int my_tok = -1;
+  float my_u = 0.f;
+  if (tid < k) {
+    my_tok = p.tokens[(size_t)b * k + tid];
+    my_u = p.u[(size_t)b * (k + 1) + tid];
+  }
+
   // ---- chunk reduction: max / first argmax, then sum of exp ----
   float vals[kMaxPerThread];
   int n = 0;
   float bv = -INFINITY;
-  int bi = 0x7fffffff;
+  int bi = INT_MAX;
   if (p.vec4) {
     const float4 *row4 = reinterpret_cast<const float4 *>(row);
 #pragma unroll
@@ -193,119 +325,147 @@ accept_stats_kernel(const __grid_constant__ AccParams p) {
       }
     }
   }
+  // the CTA whose chunk holds the draft token records its logit and q
+  const bool has_x = x_row >= c0 && x_row < c1;
+  float lx = 0.f, qx = 0.f;
+  if (has_x && tid == 0) {
+    lx = row[x_row];
+    qx = p.q[((size_t)b * k + r) * V + x_row];
+  }
   block_argmax(bv, bi, s_v, s_i);
-  double S = 0.0;
+  ff S = ff_of(0.f);
   if (!greedy && bv != -INFINITY) {
-    float acc = 0.f;
+    ff acc = ff_of(0.f);
 #pragma unroll
     for (int t = 0; t < kMaxPerThread; ++t)
-      if (t < n) acc += exp_scaled(vals[t], bv, tau);
-    S = block_sum((double)acc, s_d);
+      if (t < n) acc = ff_add(acc, ff_of(exp_scaled(vals[t], bv, tau)));
+    S = block_sum(acc, s_d);
   }
+
+  grid_dependency_wait();  // the workspace and outputs may be in use until here
   const size_t rowid = (size_t)b * (k + 1) + r;
-  if (tid == 0) p.chunks[rowid * p.C1 + c] = RowStat{bv, bi, S};
+  if (tid == 0) p.chunks[rowid * p.C1 + c] = ChunkRec{bv, bi, S, lx, qx, has_x ? 1 : 0, 0};
 
-  // ---- the last chunk of the row combines the row ----
+  // ---- the last CTA of the sequence combines every row and decides ----
   __threadfence();
   __syncthreads();
-  if (tid == 0) s_flag = (atomicAdd(p.row_tickets + rowid, 1u) == (unsigned)(p.C1 - 1));
+  if (tid == 0)
+    s_flag = (atomicAdd(p.seq_tickets + b, 1u) == (unsigned)((k + 1) * p.C1 - 1)) ? 1 : 0;
   __syncthreads();
   if (!s_flag) return;
   __threadfence();
-  float mv = -INFINITY;
-  int mi = 0x7fffffff;
-  for (int cc = tid; cc < p.C1; cc += kAccThreads) {
-    const float cm = __ldcg(&p.chunks[rowid * p.C1 + cc].m);
-    const int ca = __ldcg(&p.chunks[rowid * p.C1 + cc].arg);
-    if (better(cm, ca, mv, mi)) { mv = cm; mi = ca; }
-  }
-  block_argmax(mv, mi, s_v, s_i);
-  double Srow = 0.0;
-  if (!greedy && mv != -INFINITY) {
-    double part = 0.0;
-    for (int cc = tid; cc < p.C1; cc += kAccThreads) {
-      const float cm = __ldcg(&p.chunks[rowid * p.C1 + cc].m);
-      const double cS = __ldcg(&p.chunks[rowid * p.C1 + cc].S);
-      if (cS > 0.0) part += cS * exp(((double)cm - (double)mv) / (double)tau);
+  for (int rr = warp; rr <= k; rr += kAccWarps) {
+    const ChunkRec *cr = p.chunks + ((size_t)b * (k + 1) + rr) * p.C1;
+    float mv = -INFINITY, rlx = 0.f, rqx = 0.f;
+    int mi = INT_MAX, hx = 0;
+    for (int cc = lane; cc < p.C1; cc += 32) {
+      const float cm = __ldcg(&cr[cc].m);
+      const int ca = __ldcg(&cr[cc].arg);
+      if (better(cm, ca, mv, mi)) { mv = cm; mi = ca; }
+      if (__ldcg(&cr[cc].has_x)) {
+        hx = 1;
+        rlx = __ldcg(&cr[cc].lx);
+        rqx = __ldcg(&cr[cc].qx);
+      }
     }
-    Srow = block_sum(part, s_d);
+    warp_argmax(mv, mi);
+    const unsigned hmask = __ballot_sync(0xffffffffu, hx);
+    if (hmask) {
+      const int src = __ffs(hmask) - 1;
+      rlx = __shfl_sync(0xffffffffu, rlx, src);
+      rqx = __shfl_sync(0xffffffffu, rqx, src);
+    }
+    ff Sr = ff_of(0.f);
+    if (!greedy && mv != -INFINITY) {
+      for (int cc = lane; cc < p.C1; cc += 32) {
+        const ff cS = ff{__ldcg(&cr[cc].S.hi), __ldcg(&cr[cc].S.lo)};
+        if (ff_pos(cS))
+          Sr = ff_add(Sr, ff_mul(cS, exp_diff_accurate(__ldcg(&cr[cc].m), mv, tau)));
+      }
+      Sr = warp_sum_ff(Sr);
+    }
+    if (lane == 0) {
+      s_rm[rr] = mv;
+      s_rarg[rr] = mi;
+      s_rS[rr] = Sr;
+      s_rlx[rr] = rlx;
+      s_rqx[rr] = rqx;
+      s_rhx[rr] = hmask ? 1 : 0;
+      p.rows[(size_t)b * (k + 1) + rr] = RowStat{mv, mi, Sr};
+    }
   }
-  if (tid == 0) {
-    p.rows[rowid] = RowStat{mv, mi, Srow};
-    p.row_tickets[rowid] = 0u;
-  }
-
-  // ---- the last row of the sequence takes the k decisions ----
-  __threadfence();
   __syncthreads();
-  if (tid == 0) s_flag = (atomicAdd(p.seq_tickets + b, 1u) == (unsigned)k);
-  __syncthreads();
-  if (!s_flag) return;
-  __threadfence();
   if (tid < k) {
-    const int i = tid;
-    const int x = p.tokens[(size_t)b * k + i];
-    const RowStat rs = {__ldcg(&p.rows[(size_t)b * (k + 1) + i].m),
-                        __ldcg(&p.rows[(size_t)b * (k + 1) + i].arg),
-                        __ldcg(&p.rows[(size_t)b * (k + 1) + i].S)};
+    const int i = tid, x = my_tok;
     int acc = 0;
     float ratio = 0.f;
-    if (x < 0 || x >= V) {
+    if (x < 0 || x >= V || !s_rhx[i]) {
       set_status(p.status, SF_DEVICE_BAD_TOKEN);  // treated as a rejection
     } else if (greedy) {
-      acc = (x == rs.arg);
+      acc = (x == s_rarg[i]);
       ratio = acc ? 1.f : 0.f;
     } else {
-      const double lx = (double)__ldcg(p.logits + ((size_t)b * (k + 1) + i) * V + x);
-      const double px = exp((lx - (double)rs.m) / (double)tau) / rs.S;
-      const double qx = (double)p.q[((size_t)b * k + i) * V + x];
-      const double ux = (double)p.u[(size_t)b * (k + 1) + i];
-      acc = (ux * qx < px);
-      ratio = qx > 0.0 ? (float)fmin(1.0, px / qx) : 1.f;
+      // p(x) = exp((l_x - m) / tau) / S; accept iff u * q(x) < p(x), with the
+      // product u * q kept exactly as float-float
+      const float px = ff_div_to_f(exp_diff_accurate(s_rlx[i], s_rm[i], tau), s_rS[i]);
+      const float qd = s_rqx[i];
+      const float uq = __fmul_rn(my_u, qd);
+      const ff uqf = ff{uq, __fmaf_rn(my_u, qd, -uq)};
+      acc = ff_lt(uqf, ff_of(px)) ? 1 : 0;
+      ratio = qd > 0.f ? fminf(1.f, __fdiv_rn(px, qd)) : 1.f;
     }
     s_acc[i] = acc;
     if (p.ratio) p.ratio[(size_t)b * k + i] = ratio;
   }
   __syncthreads();
-  if (tid == 0) {
+  if (tid <= k) {
+    // every writer finds j in shared memory; thread i writes out_tokens[i]
     int j = k;
     for (int i = 0; i < k; ++i)
       if (!s_acc[i]) { j = i; break; }
-    p.num_accepted[b] = j;
-    int32_t *ob = p.out_tokens + (size_t)b * (k + 1);
-    for (int i = 0; i <= k; ++i) ob[i] = i < j ? p.tokens[(size_t)b * k + i] : -1;
-    if (greedy) ob[j] = __ldcg(&p.rows[(size_t)b * (k + 1) + j].arg);
-    p.seqs[b].j = j;
-    p.seq_tickets[b] = 0u;
+    int32_t v = -1;
+    if (tid < j) v = my_tok;
+    else if (tid == j && greedy) v = s_rarg[j];
+    if (!(tid == j && !greedy)) p.out_tokens[(size_t)b * (k + 1) + tid] = v;
+    if (tid == 0) {
+      p.num_accepted[b] = j;
+      p.seqs[b].j = j;
+      p.seq_tickets[b] = 0u;
+    }
   }
 }
 
 __global__ void __launch_bounds__(kAccThreads)
 accept_draw_kernel(const __grid_constant__ AccParams p) {
-  __shared__ double s_d[32];
-  __shared__ double s_scan[kAccThreads];
+  __shared__ ff s_d[32];
+  __shared__ ff s_scan[32];
   __shared__ float s_r[kMaxChunk];
-  __shared__ int s_flag;
-  __shared__ int s_token;
-  __shared__ int s_chunk;
-  __shared__ double s_base;
+  __shared__ int s_flag, s_token, s_chunk, s_last;
+  __shared__ ff s_base;
 
+  grid_launch_dependents();
   const int c = blockIdx.x, b = blockIdx.y;
   const int tid = threadIdx.x;
   const int k = p.k, V = p.V;
   const float tau = p.tau[b];
   if (!(tau > 0.0f)) return;  // greedy sequences are complete
-  const int j = p.seqs[b].j;
+  const float u_k = p.u[(size_t)b * (k + 1) + k];
+  grid_dependency_wait();     // j and the row statistics come from the previous kernel
+
+  const int j = __ldcg(&p.seqs[b].j);
+  const RowStat rs = {__ldcg(&p.rows[(size_t)b * (k + 1) + j].m),
+                      __ldcg(&p.rows[(size_t)b * (k + 1) + j].arg),
+                      ff{__ldcg(&p.rows[(size_t)b * (k + 1) + j].S.hi),
+                         __ldcg(&p.rows[(size_t)b * (k + 1) + j].S.lo)}};
   const bool residual = j < k;
-  const RowStat rs = p.rows[(size_t)b * (k + 1) + j];
-  const float invS = (float)(1.0 / rs.S);
+  const float invS = ff_div_to_f(1.0f, rs.S);
   const float *row = p.logits + ((size_t)b * (k + 1) + j) * V;
   const float *qrow = residual ? p.q + ((size_t)b * k + j) * V : nullptr;
   const int c0 = c * p.CV2;
   const int c1 = min(V, c0 + p.CV2);
 
-  // ---- chunk sums of r and p (fp32 per thread, fp64 across threads) ----
-  float sr = 0.f, sp = 0.f;
+  // ---- chunk sums of r and p (float-float) ----
+  ff sr = ff_of(0.f), sp = ff_of(0.f);
   int lr = -1, lp = -1;
   if (p.vec4) {
     for (int e = c0 + 4 * tid; e < c1; e += 4 * kAccThreads) {
@@ -318,8 +478,8 @@ accept_draw_kernel(const __grid_constant__ AccParams p) {
       for (int t = 0; t < 4; ++t) {
         float rr, pz;
         draw_terms(xs[t], qs[t], residual, rs.m, tau, invS, rr, pz);
-        sr += rr;
-        sp += pz;
+        sr = ff_add(sr, ff_of(rr));
+        sp = ff_add(sp, ff_of(pz));
         if (rr > 0.f) lr = e + t;
         if (pz > 0.f) lp = e + t;
       }
@@ -328,21 +488,21 @@ accept_draw_kernel(const __grid_constant__ AccParams p) {
     for (int e = c0 + tid; e < c1; e += kAccThreads) {
       float rr, pz;
       draw_terms(row[e], residual ? qrow[e] : 0.f, residual, rs.m, tau, invS, rr, pz);
-      sr += rr;
-      sp += pz;
+      sr = ff_add(sr, ff_of(rr));
+      sp = ff_add(sp, ff_of(pz));
       if (rr > 0.f) lr = e;
       if (pz > 0.f) lp = e;
     }
   }
-  const double Sr = block_sum((double)sr, s_d);
-  const double Sp = block_sum((double)sp, s_d);
+  const ff Sr = block_sum(sr, s_d);
+  const ff Sp = block_sum(sp, s_d);
   {
-    int v = lr;
+    int v = lr, w = lp;
 #pragma unroll
-    for (int o = 16; o > 0; o >>= 1) v = max(v, __shfl_xor_sync(0xffffffffu, v, o));
-    int w = lp;
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) w = max(w, __shfl_xor_sync(0xffffffffu, w, o));
+    for (int o = 16; o > 0; o >>= 1) {
+      v = max(v, __shfl_xor_sync(0xffffffffu, v, o));
+      w = max(w, __shfl_xor_sync(0xffffffffu, w, o));
+    }
     if (tid == 0) { s_flag = -1; s_token = -1; }
     __syncthreads();
     if ((tid & 31) == 0) { atomicMax(&s_flag, v); atomicMax(&s_token, w); }
@@ -353,67 +513,63 @@ accept_draw_kernel(const __grid_constant__ AccParams p) {
   // ---- the last chunk of the sequence draws the token ----
   __threadfence();
   __syncthreads();
-  if (tid == 0) s_flag = (atomicAdd(p.draw_tickets + b, 1u) == (unsigned)(p.C2 - 1));
+  if (tid == 0) s_flag = (atomicAdd(p.draw_tickets + b, 1u) == (unsigned)(p.C2 - 1)) ? 1 : 0;
   __syncthreads();
   if (!s_flag) return;
   __threadfence();
 
   const DrawPart *parts = p.parts + (size_t)b * p.C2;
-  double total = 0.0;
+  auto part_sum = [&](int cc, bool pmass) -> ff {
+    return pmass ? ff{__ldcg(&parts[cc].sum_p.hi), __ldcg(&parts[cc].sum_p.lo)}
+                 : ff{__ldcg(&parts[cc].sum_r.hi), __ldcg(&parts[cc].sum_r.lo)};
+  };
+  ff total;
   {
-    double pr = 0.0;
-    for (int cc = tid; cc < p.C2; cc += kAccThreads) pr += __ldcg(&parts[cc].sum_r);
+    ff pr = ff_of(0.f);
+    for (int cc = tid; cc < p.C2; cc += kAccThreads) pr = ff_add(pr, part_sum(cc, false));
     total = block_sum(pr, s_d);
   }
-  const bool use_p = !(total > 0.0);  // residual with no mass (rounding only)
+  const bool use_p = !ff_pos(total);  // residual with no mass (rounding only)
   if (use_p) {
-    double pp = 0.0;
-    for (int cc = tid; cc < p.C2; cc += kAccThreads) pp += __ldcg(&parts[cc].sum_p);
+    ff pp = ff_of(0.f);
+    for (int cc = tid; cc < p.C2; cc += kAccThreads) pp = ff_add(pp, part_sum(cc, true));
     total = block_sum(pp, s_d);
   }
-  const double target = (double)p.u[(size_t)b * (k + 1) + k] * total;
+  const ff target = ff_mul(total, u_k);
 
-  // chunk holding the target: inclusive fp64 scan over chunk sums, in order
-  if (tid == 0) { s_chunk = 0x7fffffff; s_base = 0.0; }
-  double carry = 0.0;
+  // chunk holding the target: inclusive fp64 scan over chunk sums in order;
+  // chunk cc covers [excl, incl), and excl of cc is bit-identical to incl of
+  // cc - 1, so the intervals tile [0, total) without gaps or overlaps
+  if (tid == 0) { s_chunk = INT_MAX; s_base = ff_of(0.f); }
+  ff carry = ff_of(0.f);
   for (int base = 0; base < p.C2; base += kAccThreads) {
     const int cc = base + tid;
-    double v = 0.0;
-    if (cc < p.C2) v = use_p ? __ldcg(&parts[cc].sum_p) : __ldcg(&parts[cc].sum_r);
+    const ff v = cc < p.C2 ? part_sum(cc, use_p) : ff_of(0.f);
+    ff excl_local, blk_total;
+    const ff incl_local = block_inclusive_scan(v, s_scan, &excl_local, &blk_total);
+    const ff excl = ff_add(carry, excl_local), incl = ff_add(carry, incl_local);
+    if (cc < p.C2 && ff_pos(v) && ff_lt(target, incl) && !ff_lt(target, excl))
+      atomicMin(&s_chunk, cc);
     __syncthreads();
-    s_scan[tid] = v;
+    if (s_chunk == cc) s_base = excl;
+    carry = ff_add(carry, blk_total);
     __syncthreads();
-    for (int o = 1; o < kAccThreads; o <<= 1) {
-      const double add = tid >= o ? s_scan[tid - o] : 0.0;
-      __syncthreads();
-      s_scan[tid] += add;
-      __syncthreads();
-    }
-    // excl of chunk cc is bit-identical to incl of chunk cc-1, so the chunk
-    // intervals [excl, incl) tile [0, total) without gaps or overlaps
-    const double incl = carry + s_scan[tid];
-    const double excl = carry + (tid > 0 ? s_scan[tid - 1] : 0.0);
-    if (cc < p.C2 && v > 0.0 && target < incl && target >= excl) atomicMin(&s_chunk, cc);
-    __syncthreads();
-    if (s_chunk == cc && cc < p.C2) s_base = excl;
-    carry += s_scan[kAccThreads - 1];
-    __syncthreads();
-    if (s_chunk != 0x7fffffff) break;
+    if (s_chunk != INT_MAX) break;
   }
   __syncthreads();
   int token = -1;
-  if (s_chunk == 0x7fffffff) {
+  if (s_chunk == INT_MAX) {
     // u*S at or past the total (rounding): the last token with positive mass
     int last = -1;
     for (int cc = tid; cc < p.C2; cc += kAccThreads)
       last = max(last, use_p ? __ldcg(&parts[cc].last_p) : __ldcg(&parts[cc].last_r));
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) last = max(last, __shfl_xor_sync(0xffffffffu, last, o));
-    if (tid == 0) s_token = -1;
+    if (tid == 0) s_last = -1;
     __syncthreads();
-    if ((tid & 31) == 0) atomicMax(&s_token, last);
+    if ((tid & 31) == 0) atomicMax(&s_last, last);
     __syncthreads();
-    token = s_token;
+    token = s_last;
   } else {
     // scan the chunk in ascending token order: thread t owns a contiguous run
     const int cc = s_chunk;
@@ -427,26 +583,20 @@ accept_draw_kernel(const __grid_constant__ AccParams p) {
     __syncthreads();
     const int per = (len + kAccThreads - 1) / kAccThreads;
     const int a0 = tid * per, a1 = min(len, a0 + per);
-    double mine = 0.0;
-    for (int e = a0; e < a1; ++e) mine += (double)s_r[e];
-    s_scan[tid] = mine;
-    __syncthreads();
-    for (int o = 1; o < kAccThreads; o <<= 1) {
-      const double add = tid >= o ? s_scan[tid - o] : 0.0;
-      __syncthreads();
-      s_scan[tid] += add;
-      __syncthreads();
-    }
-    double cum = s_base + (tid > 0 ? s_scan[tid - 1] : 0.0);
-    if (tid == 0) s_token = 0x7fffffff;
+    ff mine = ff_of(0.f);
+    for (int e = a0; e < a1; ++e) mine = ff_add(mine, ff_of(s_r[e]));
+    ff excl, unused;
+    block_inclusive_scan(mine, s_scan, &excl, &unused);
+    ff cum = ff_add(s_base, excl);
+    if (tid == 0) s_token = INT_MAX;
     __syncthreads();
     for (int e = a0; e < a1; ++e) {
-      cum += (double)s_r[e];
-      if (target < cum) { atomicMin(&s_token, e0 + e); break; }
+      cum = ff_add(cum, ff_of(s_r[e]));
+      if (ff_lt(target, cum)) { atomicMin(&s_token, e0 + e); break; }
     }
     __syncthreads();
     token = s_token;
-    if (token == 0x7fffffff) {
+    if (token == INT_MAX) {
       // rounding put the target past this chunk's own sum: its last positive token
       token = use_p ? __ldcg(&parts[cc].last_p) : __ldcg(&parts[cc].last_r);
     }
@@ -465,7 +615,7 @@ struct AccPlan {
 };
 
 struct AccLayout {
-  size_t row_tickets, seq_tickets, draw_tickets, rows, chunks, seqs, parts, total;
+  size_t seq_tickets, draw_tickets, chunks, rows, seqs, parts, total;
 };
 
 static int chunking(long long target_ctas, int V, int rows, int *C, int *CV) {
@@ -497,11 +647,10 @@ static AccLayout acc_layout(int B, int k, const AccPlan &pl) {
   AccLayout l;
   const size_t R = (size_t)B * (k + 1);
   size_t off = 256;
-  l.row_tickets = off; off = round_up(off + 4 * R, 256);
   l.seq_tickets = off; off = round_up(off + 4 * (size_t)B, 256);
   l.draw_tickets = off; off = round_up(off + 4 * (size_t)B, 256);
+  l.chunks = off; off = round_up(off + sizeof(ChunkRec) * R * pl.C1, 256);
   l.rows = off; off = round_up(off + sizeof(RowStat) * R, 256);
-  l.chunks = off; off = round_up(off + sizeof(RowStat) * R * pl.C1, 256);
   l.seqs = off; off = round_up(off + sizeof(SeqState) * (size_t)B, 256);
   l.parts = off; off = round_up(off + sizeof(DrawPart) * (size_t)B * pl.C2, 256);
   l.total = off;
@@ -563,11 +712,10 @@ int sf_accept(const float *target_logits, const float *draft_probs,
   prm.out_tokens = out_tokens;
   prm.ratio = accept_ratio;
   prm.status = reinterpret_cast<uint32_t *>(ws);
-  prm.row_tickets = reinterpret_cast<uint32_t *>(ws + lay.row_tickets);
   prm.seq_tickets = reinterpret_cast<uint32_t *>(ws + lay.seq_tickets);
   prm.draw_tickets = reinterpret_cast<uint32_t *>(ws + lay.draw_tickets);
+  prm.chunks = reinterpret_cast<ChunkRec *>(ws + lay.chunks);
   prm.rows = reinterpret_cast<RowStat *>(ws + lay.rows);
-  prm.chunks = reinterpret_cast<RowStat *>(ws + lay.chunks);
   prm.seqs = reinterpret_cast<SeqState *>(ws + lay.seqs);
   prm.parts = reinterpret_cast<DrawPart *>(ws + lay.parts);
   prm.B = B;
@@ -579,11 +727,23 @@ int sf_accept(const float *target_logits, const float *draft_probs,
   prm.CV2 = plan.CV2;
   prm.vec4 = (V % 4 == 0) && aligned(target_logits, 16) && aligned(draft_probs, 16);
 
-  accept_stats_kernel<<<dim3(plan.C1, k + 1, B), kAccThreads, 0, stream>>>(prm);
-  cudaError_t e = cudaGetLastError();
+  // Both kernels are launched with programmatic stream serialisation: each
+  // may be scheduled while the previous kernel on the stream drains and
+  // waits for it (griddepcontrol.wait) before writing or reading its results.
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(plan.C1, k + 1, B);
+  cfg.blockDim = dim3(kAccThreads);
+  cfg.dynamicSmemBytes = 0;
+  cfg.stream = stream;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  cudaError_t e = cudaLaunchKernelEx(&cfg, accept_stats_kernel, prm);
   if (e != cudaSuccess) return fail(SF_ERR_CUDA, "accept stats launch: %s", cudaGetErrorString(e));
-  accept_draw_kernel<<<dim3(plan.C2, B), kAccThreads, 0, stream>>>(prm);
-  e = cudaGetLastError();
+  cfg.gridDim = dim3(plan.C2, B);
+  e = cudaLaunchKernelEx(&cfg, accept_draw_kernel, prm);
   if (e != cudaSuccess) return fail(SF_ERR_CUDA, "accept draw launch: %s", cudaGetErrorString(e));
   return SF_OK;
 }
