@@ -171,6 +171,17 @@ __device__ __forceinline__ float4 ld_dsmem_f32x4(uint32_t local, uint32_t rank) 
   return v;
 }
 
+// Stores into the shared memory of another CTA of the cluster (an address
+// obtained with dsmem_addr).
+__device__ __forceinline__ void st_dsmem_f32(uint32_t remote, float v) {
+  asm volatile("st.shared::cluster.f32 [%0], %1;" ::"r"(remote), "f"(v) : "memory");
+}
+
+__device__ __forceinline__ void st_dsmem_f32x2(uint32_t remote, float a, float b) {
+  asm volatile("st.shared::cluster.v2.f32 [%0], {%1, %2};" ::"r"(remote), "f"(a), "f"(b)
+               : "memory");
+}
+
 __device__ __forceinline__ void set_status(uint32_t *status, uint32_t bits) {
   atomicOr(status, bits);
 }

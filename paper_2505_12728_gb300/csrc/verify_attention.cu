@@ -65,6 +65,8 @@ struct AttnParams {
   uint32_t *tickets;  // [B * H_kv], zero between calls (in-kernel merge)
   int merge_in_kernel;  // 1: last CTA of a segment merges; 0: merge kernel
   int cs;             // CTAs per cluster of the launch (1: no clusters)
+  int push;           // cluster mode: peers push partial rows into the merging CTA
+  int push_off;       // byte offset of the push area in dynamic shared memory
   float *partials;    // [G + B * H_kv][R][D + 2]
   int B, n_q, H_q, H_kv, group, R;
   int num_pages, max_pages, max_tokens;
@@ -154,6 +156,7 @@ __device__ __forceinline__ int owner_cta(long long t, long long Tot, int G) {
 
 constexpr int kMergeBatch = 16;
 constexpr int kMaxCluster = 16;  // largest cluster launched (non-portable size)
+constexpr int kPushSlots = 2;    // rows a CTA merges in push mode (at most)
 
 template <bool kBypassL1, typename T>
 __device__ __forceinline__ T merge_load(const T *p) {
@@ -517,9 +520,9 @@ verify_attention_kernel(const __grid_constant__ CUtensorMap tmap_k,
           (void)mbar_wait_bounded(bar0 + 8 * (x % STAGES), (x / STAGES) & 1u);
       }
       __syncthreads();
-      if (aligned) {  // the cluster's other CTAs expect two barrier arrivals
+      if (aligned) {  // the cluster's other CTAs expect this CTA's barrier arrivals
         cluster_sync();
-        cluster_sync();
+        if (!p.push) cluster_sync();
       }
       return;
     }
@@ -614,6 +617,30 @@ verify_attention_kernel(const __grid_constant__ CUtensorMap tmap_k,
       continue;
     }
 
+    if (aligned && p.push) {
+      // push each partial row into the shared memory of the CTA that merges
+      // it: rank rho merges rows [rho*R/cs, (rho+1)*R/cs); entry
+      // [row slot][sender rank] holds O (D floats), m, l (stride D + 4)
+      const int cs = p.cs, rank = static_cast<int>(blockIdx.x) % cs;
+      auto push_row = [&](int r, const float (&oo)[DT][4], int h, float mm, float ll) {
+        const int rho = ((r + 1) * cs - 1) / p.R;
+        const int slot = r - rho * p.R / cs;
+        const uint32_t entry = ring + p.push_off + 4u * ((slot * cs + rank) * (D + 4));
+        const uint32_t remote = dsmem_addr(entry, rho);
+#pragma unroll
+        for (int dt = 0; dt < DT; ++dt)
+          st_dsmem_f32x2(remote + 4u * (dt * 8 + colb), oo[dt][2 * h], oo[dt][2 * h + 1]);
+        if ((lane & 3) == 0) {
+          st_dsmem_f32(remote + 4u * D, mm);
+          st_dsmem_f32(remote + 4u * (D + 1), ll);
+        }
+      };
+      if (writer) {
+        if (r0 < p.R) push_row(r0, o, 0, m0, l0);
+        if (r1 < p.R) push_row(r1, o, 1, m1, l1);
+      }
+      continue;
+    }
     if (aligned) {
       // partial of this CTA's piece into its own shared memory (ring, idle):
       // O [R][D] fp32, then m [R], l [R]; read by the cluster after the barrier
@@ -697,7 +724,39 @@ verify_attention_kernel(const __grid_constant__ CUtensorMap tmap_k,
     }
     __syncthreads();
   }
-  if (aligned) {
+  if (aligned && p.push) {
+    // Every peer has pushed its rows; merge this CTA's rows from its own
+    // shared memory, in rank order (= tile order).  Nobody reads this CTA's
+    // shared memory, so there is no second barrier.
+    cluster_sync();
+    const int cs = p.cs, rank = static_cast<int>(blockIdx.x) % cs;
+    const int R = p.R;
+    const int r_lo = rank * R / cs, r_hi = (rank + 1) * R / cs;
+    const float *push = reinterpret_cast<const float *>(smem + p.push_off);
+    for (int idx = tid; idx < (r_hi - r_lo) * (D / 4); idx += NTHREADS) {
+      const int slot = idx / (D / 4), c4 = idx % (D / 4);
+      const int r = r_lo + slot;
+      float M = -INFINITY;
+      for (int u = 0; u < cs; ++u) M = fmaxf(M, push[(slot * cs + u) * (D + 4) + D]);
+      float Ls = 0.f;
+      float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+      for (int u = 0; u < cs; ++u) {
+        const float *e = push + (slot * cs + u) * (D + 4);
+        const float w = exp2f(e[D] - M);
+        Ls += e[D + 1] * w;
+        const float4 x = *reinterpret_cast<const float4 *>(e + 4 * c4);
+        acc.x += x.x * w; acc.y += x.y * w; acc.z += x.z * w; acc.w += x.w * w;
+      }
+      const float inv = 1.f / Ls;
+      const int i = r / p.group, j = r % p.group;
+      const size_t row = ((size_t)seg_b * p.n_q + i) * p.H_q + (size_t)seg_h * p.group + j;
+      uint2 packed;
+      packed.x = pack_bf16x2(acc.x * inv, acc.y * inv);
+      packed.y = pack_bf16x2(acc.z * inv, acc.w * inv);
+      *reinterpret_cast<uint2 *>(p.out + row * D + 4 * c4) = packed;
+      if (p.lse && c4 == 0) p.lse[row] = (M + log2f(Ls)) * kLn2;
+    }
+  } else if (aligned) {
     // Every CTA's partial is in its shared memory; CTA `rank` of the cluster
     // merges rows [rank*R/cs, (rank+1)*R/cs) over the cluster's pieces, which
     // are in rank order (= tile order), reading them through distributed
@@ -797,6 +856,7 @@ struct AttnVariant {
   int threads;
   int stages;
   int smem_fixed;  // bytes excluding the per-batch arrays
+  int prefix_off;  // byte offset of the per-batch arrays in shared memory
   int ks, nw;
 };
 
@@ -808,6 +868,7 @@ static AttnVariant make_variant() {
   v.threads = NW * 32;
   v.stages = STAGES;
   v.smem_fixed = AttnSmem<D, STAGES, NW>::bytes(0);
+  v.prefix_off = AttnSmem<D, STAGES, NW>::kPrefixOffset;
   v.ks = KS;
   v.nw = NW;
   return v;
@@ -862,8 +923,16 @@ struct AttnPlan {
   AttnVariant v;
   int G;
   int smem;
-  int cs;  // CTAs per cluster (1: no clusters)
+  int cs;        // CTAs per cluster (1: no clusters)
+  int push;      // cluster mode pushes partial rows (few rows per merging CTA)
+  int push_off;  // byte offset of the push area in shared memory
 };
+
+// Largest dynamic shared memory a launch of variant v can ask for: the
+// per-batch arrays at SF_MAX_BATCH plus a full push area.
+static int max_dynamic_smem(const AttnVariant &v) {
+  return v.smem_fixed + 8 * SF_MAX_BATCH + 16 + kPushSlots * kMaxCluster * (128 + 4) * 4;
+}
 
 // Per-device, per-kernel launch facts, computed once: the dynamic shared
 // memory limit is raised to the largest size any batch needs, and resident
@@ -876,7 +945,7 @@ static int kernel_setup(const AttnVariant &v, int dev, int smem, int *occ_out) {
   void *key = reinterpret_cast<void *>(v.fn);
   if (!attr_done[{key, dev}]) {
     cudaError_t e = cudaFuncSetAttribute(v.fn, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         v.smem_fixed + 8 * SF_MAX_BATCH);
+                                         max_dynamic_smem(v));
     if (e != cudaSuccess) return fail(SF_ERR_CUDA, "cudaFuncSetAttribute: %s", cudaGetErrorString(e));
     attr_done[{key, dev}] = true;
   }
@@ -939,9 +1008,11 @@ static int plan_attention(int B, int n_q, int H_q, int H_kv, int D, int max_page
   const int R = n_q * (H_q / H_kv);
   plan->v = select_variant(D, R);
   plan->smem = plan->v.smem_fixed + 8 * B;
-  if (plan->v.smem_fixed + 8 * SF_MAX_BATCH > dev.max_smem_optin)
+  plan->push = 0;
+  plan->push_off = 0;
+  if (max_dynamic_smem(plan->v) > dev.max_smem_optin)
     return fail(SF_ERR_UNSUPPORTED, "needs %d B shared memory, device allows %d",
-                plan->v.smem_fixed + 8 * SF_MAX_BATCH, dev.max_smem_optin);
+                max_dynamic_smem(plan->v), dev.max_smem_optin);
   int occ = 1;
   st = kernel_setup(plan->v, dev.ordinal, plan->smem, &occ);
   if (st != SF_OK) return st;
@@ -973,6 +1044,12 @@ static int plan_attention(int B, int n_q, int H_q, int H_kv, int D, int max_page
   if (G > max_tiles) G = max_tiles;
   if (G > (1 << 20)) G = 1 << 20;
   plan->G = static_cast<int>(G < 1 ? 1 : G);
+  if (plan->cs > 1 && (R + plan->cs - 1) / plan->cs <= kPushSlots) {
+    // push area after the per-batch arrays: kPushSlots x cs entries of D + 4 floats
+    plan->push = 1;
+    plan->push_off = static_cast<int>(round_up((size_t)plan->v.prefix_off + 4 * (2 * B + 2), 16));
+    plan->smem = plan->push_off + 1024 + kPushSlots * plan->cs * (D + 4) * 4;
+  }
   return SF_OK;
 }
 
@@ -1078,6 +1155,8 @@ int sf_verify_attention(const void *q, const void *k_cache, const void *v_cache,
   // grid-wide merge kernel spreads the larger partials over many SMs.
   prm.merge_in_kernel = R <= 16 ? 1 : 0;
   prm.cs = plan.cs;
+  prm.push = plan.push;
+  prm.push_off = plan.push_off;
   prm.partials = reinterpret_cast<float *>(ws + lay.partials_off);
   prm.B = B;
   prm.n_q = n_q;
