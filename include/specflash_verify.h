@@ -109,8 +109,9 @@ int sf_read_device_status(const void *workspace, uint32_t *status_out);
 /*              H_q / H_kv <= 8; 1 <= B <= 1024.                             */
 /* softmax_scale  0 selects 1/sqrt(head_dim).                                */
 /* num_splits   number of cooperating CTAs the batch's KV tiles are divided */
-/*              among; 0 picks (SM count x resident CTAs per SM).  The        */
-/*              result depends on it only through rounding.                 */
+/*              among (at most 65535); 0 picks the grid from the SM count    */
+/*              (and, for one sequence, one thread-block cluster per KV      */
+/*              head).  The result depends on it only through rounding.      */
 /* out          bf16 [B][n_q][H_q][head_dim].                                */
 /* lse          fp32 [B][n_q][H_q] (natural log, scaled scores); may be NULL.*/
 /* workspace    >= sf_verify_attention_workspace_size(...) bytes, 256-byte   */

@@ -139,22 +139,35 @@ __device__ void tile_prefix(const AttnParams &p, int *s_prefix, int *s_len, int 
   if (tid == NT - 1) s_prefix[p.B] = warp_off + incl;
 }
 
+// The tile partition uses 32-bit arithmetic only (the host guarantees
+// fewer than 2^31 tiles and G <= 65535): CTA c owns the global tiles
+// [start(c), start(c+1)) with start(c) = floor(c * Tot / G), computed as
+// c*q + floor(c*r / G) with q = Tot / G, r = Tot % G (c*r < G^2 < 2^32).
+struct TilePartition {
+  uint32_t Tot, G, q, r;
+  __device__ __forceinline__ uint32_t start(uint32_t c) const { return c * q + (c * r) / G; }
+  // CTA whose range contains tile t: an fp32 estimate, then exact steps
+  __device__ __forceinline__ uint32_t owner(uint32_t t) const {
+    int c = static_cast<int>((static_cast<float>(t) + 0.5f) * (static_cast<float>(G) / static_cast<float>(Tot)));
+    c = c < 0 ? 0 : (c >= static_cast<int>(G) ? static_cast<int>(G) - 1 : c);
+    while (c > 0 && start(static_cast<uint32_t>(c)) > t) --c;
+    while (c + 1 < static_cast<int>(G) && start(static_cast<uint32_t>(c + 1)) <= t) ++c;
+    return static_cast<uint32_t>(c);
+  }
+};
+
 // Sequence b owning global tile t: H_kv * s_prefix[b] <= t < H_kv * s_prefix[b+1].
-__device__ __forceinline__ int find_sequence(long long t, const int *s_prefix, int B, int H_kv) {
+__device__ __forceinline__ int find_sequence(uint32_t t, const int *s_prefix, int B, int H_kv) {
   int lo = 0, hi = B - 1;
   while (lo < hi) {
     int mid = (lo + hi + 1) >> 1;
-    if ((long long)H_kv * s_prefix[mid] <= t) lo = mid; else hi = mid - 1;
+    if (static_cast<uint32_t>(H_kv) * static_cast<uint32_t>(s_prefix[mid]) <= t) lo = mid; else hi = mid - 1;
   }
   return lo;
 }
 
-// CTA whose range [c*Tot/G, (c+1)*Tot/G) contains global tile t.
-__device__ __forceinline__ int owner_cta(long long t, long long Tot, int G) {
-  return static_cast<int>(((t + 1) * G - 1) / Tot);
-}
-
 constexpr int kMergeBatch = 16;
+constexpr int kMaxGrid = 65535;  // CTAs of one launch (the partition uses 32-bit math)
 constexpr int kMaxCluster = 16;  // largest cluster launched (non-portable size)
 constexpr int kPushSlots = 2;    // rows a CTA merges in push mode (at most)
 
@@ -256,11 +269,12 @@ verify_attention_kernel(const __grid_constant__ CUtensorMap tmap_k,
   // CTAs than tiles the surplus CTAs leave, so that every CTA of the
   // partition owns at least one tile and a segment's pieces are owned by
   // consecutive CTAs.
-  const long long Tot = (long long)p.H_kv * s_prefix[p.B];
-  const int G = Tot < (long long)p.G ? static_cast<int>(Tot) : p.G;
+  const uint32_t Tot = static_cast<uint32_t>(p.H_kv) * static_cast<uint32_t>(s_prefix[p.B]);
+  const int G = Tot < static_cast<uint32_t>(p.G) ? static_cast<int>(Tot) : p.G;
   if (static_cast<int>(blockIdx.x) >= G) return;
-  const long long t_begin = (long long)blockIdx.x * Tot / G;
-  const long long t_end = (long long)(blockIdx.x + 1) * Tot / G;
+  const TilePartition part_of{Tot, static_cast<uint32_t>(G), Tot / G, Tot % G};
+  const uint32_t t_begin = part_of.start(blockIdx.x);
+  const uint32_t t_end = part_of.start(blockIdx.x + 1);
 
   // Cluster mode: when the launch uses clusters of cs CTAs and a cluster's
   // tiles are exactly one segment (uniform segments with G = segments x cs),
@@ -270,11 +284,11 @@ verify_attention_kernel(const __grid_constant__ CUtensorMap tmap_k,
   // every CTA of an aligned cluster has exactly one piece.
   bool aligned = false;
   if (p.cs > 1 && G == p.G) {
-    const long long k = blockIdx.x / p.cs;
-    const long long c0 = k * p.cs * Tot / G, c1 = (k + 1) * p.cs * Tot / G;
+    const uint32_t k = blockIdx.x / p.cs;
+    const uint32_t c0 = part_of.start(k * p.cs), c1 = part_of.start((k + 1) * p.cs);
     const int bb = find_sequence(c0, s_prefix, p.B, p.H_kv);
-    const int tb = s_prefix[bb + 1] - s_prefix[bb];
-    const long long base = (long long)p.H_kv * s_prefix[bb];
+    const uint32_t tb = static_cast<uint32_t>(s_prefix[bb + 1] - s_prefix[bb]);
+    const uint32_t base = static_cast<uint32_t>(p.H_kv) * static_cast<uint32_t>(s_prefix[bb]);
     aligned = ((c0 - base) % tb == 0) && (c1 - c0 == tb);
   }
   int seg_b = 0, seg_h = 0;  // the segment of an aligned cluster
@@ -284,19 +298,19 @@ verify_attention_kernel(const __grid_constant__ CUtensorMap tmap_k,
   uint32_t consumed = 0;  // tiles consumed by this CTA so far (ring position)
   bool timed_out = false;
 
-  for (long long t = t_begin; t < t_end && !timed_out;) {
+  for (uint32_t t = t_begin; t < t_end && !timed_out;) {
     // ---- locate the piece: segment (b, h_kv), local tiles [lt0, lt1) ----
     const int b = find_sequence(t, s_prefix, p.B, p.H_kv);
     const int tiles_b = s_prefix[b + 1] - s_prefix[b];
-    const long long seg_base = (long long)p.H_kv * s_prefix[b];
-    const int h_kv = static_cast<int>((t - seg_base) / tiles_b);
-    const int lt0 = static_cast<int>((t - seg_base) % tiles_b);
-    const long long left = t_end - t;
-    const int n_tiles = left < (long long)(tiles_b - lt0) ? static_cast<int>(left) : tiles_b - lt0;
-    const long long seg_first = seg_base + (long long)h_kv * tiles_b;
+    const uint32_t seg_base = static_cast<uint32_t>(p.H_kv) * static_cast<uint32_t>(s_prefix[b]);
+    const int h_kv = static_cast<int>((t - seg_base) / static_cast<uint32_t>(tiles_b));
+    const int lt0 = static_cast<int>((t - seg_base) % static_cast<uint32_t>(tiles_b));
+    const uint32_t left = t_end - t;
+    const int n_tiles = left < static_cast<uint32_t>(tiles_b - lt0) ? static_cast<int>(left) : tiles_b - lt0;
+    const uint32_t seg_first = seg_base + static_cast<uint32_t>(h_kv) * static_cast<uint32_t>(tiles_b);
     const int seg = b * p.H_kv + h_kv;
-    const int c_first = owner_cta(seg_first, Tot, G);
-    const int c_last = owner_cta(seg_first + tiles_b - 1, Tot, G);
+    const int c_first = static_cast<int>(part_of.owner(seg_first));
+    const int c_last = static_cast<int>(part_of.owner(seg_first + tiles_b - 1));
     const int n_pieces = c_last - c_first + 1;
     const int T = s_len[b];
     const int Lb = T - p.n_q;
@@ -1018,6 +1032,8 @@ static int plan_attention(int B, int n_q, int H_q, int H_kv, int D, int max_page
   if (st != SF_OK) return st;
   const long long max_tiles =
       (long long)B * H_kv * (((long long)max_pages_per_seq * SF_PAGE_SIZE + kTileTokens - 1) / kTileTokens);
+  if (max_tiles >= (1LL << 31))
+    return fail(SF_ERR_UNSUPPORTED, "B x H_kv x tiles per sequence = %lld tiles (limit 2^31)", max_tiles);
   const long long capacity = (long long)dev.sm_count * occ;
   long long G = num_splits > 0 ? num_splits : capacity;
   plan->cs = 1;
@@ -1042,7 +1058,7 @@ static int plan_attention(int B, int n_q, int H_q, int H_kv, int D, int max_page
     }
   }
   if (G > max_tiles) G = max_tiles;
-  if (G > (1 << 20)) G = 1 << 20;
+  if (G > kMaxGrid) G = kMaxGrid;
   plan->G = static_cast<int>(G < 1 ? 1 : G);
   if (plan->cs > 1 && (R + plan->cs - 1) / plan->cs <= kPushSlots) {
     // push area after the per-batch arrays: kPushSlots x cs entries of D + 4 floats
