@@ -3,9 +3,9 @@
  * SpecFLASH speculative decoding (arXiv 2505.12728).
  *
  * The verification step has two parts (Sec. 3.1, "Preliminaries"; Sec. 3.3):
- *   1. the target model scores the K draft tokens "in parallel within a single
- *      forward pass": per layer, attention of the K new query rows over the
- *      cached (mostly visual) prefix plus the causal draft block
+ *   1. the target model scores all K draft tokens together, in one forward
+ *      pass: per layer, attention of the K new query rows over the cached
+ *      (mostly visual) prefix plus the causal draft block
  *      (sf_verify_attention);
  *   2. the token-wise acceptance-rejection rule: candidate T'_i is kept with
  *      probability min(1, p_i/q_i), candidates after the first rejection are
@@ -33,6 +33,13 @@
  *     workspaces.  Re-initialise after a nonzero device status.
  *   - Results are deterministic: for fixed shapes, inputs and num_splits they
  *     are bit-identical from run to run (no floating-point atomics).
+ *   - Stream order: kernels are launched with programmatic dependent launch,
+ *     so each may start while the previous kernel on `stream` drains.  Before
+ *     waiting for that kernel, sf_verify_attention reads the block table, the
+ *     sequence lengths and the prefix part of the KV cache (positions below
+ *     seq_lens[b] - n_q); these, and the workspace, must not be written by
+ *     the kernel immediately before it on the stream.  Everything else (q,
+ *     the draft rows' K/V, logits, probabilities, tokens, uniforms) may be.
  */
 #ifndef SPECFLASH_VERIFY_H
 #define SPECFLASH_VERIFY_H
@@ -86,9 +93,9 @@ int sf_workspace_init(void *workspace, size_t bytes, cudaStream_t stream);
 int sf_read_device_status(const void *workspace, uint32_t *status_out);
 
 /* ------------------------------------------------------------------------ */
-/* Verification attention (Sec. 3.1: "computes the probabilities of these K  */
-/* candidate tokens in parallel within a single forward pass"; the verify    */
-/* costs about one target step, Eq. 1).                                      */
+/* Verification attention (Sec. 3.1: the K candidates' probabilities come  */
+/* from one parallel forward pass of the target model; the verify costs     */
+/* about one target step, Eq. 1).                                            */
 /*                                                                           */
 /* For each sequence b, draft row i < n_q and query head h (KV head          */
 /* h / (H_q / H_kv)): the visible keys are the L_b = seq_lens[b] - n_q       */
@@ -111,7 +118,10 @@ int sf_read_device_status(const void *workspace, uint32_t *status_out);
 /* num_splits   number of cooperating CTAs the batch's KV tiles are divided */
 /*              among (at most 65535); 0 picks the grid from the SM count    */
 /*              (and, for one sequence, one thread-block cluster per KV      */
-/*              head).  The result depends on it only through rounding.      */
+/*              head).  With more than 16 rows per KV head                   */
+/*              (n_q * H_q / H_kv > 16) the tcgen05 kernel runs one CTA per  */
+/*              SM and uses min(num_splits, SM count) CTAs.  The result      */
+/*              depends on it only through rounding.                         */
 /* out          bf16 [B][n_q][H_q][head_dim].                                */
 /* lse          fp32 [B][n_q][H_q] (natural log, scaled scores); may be NULL.*/
 /* workspace    >= sf_verify_attention_workspace_size(...) bytes, 256-byte   */

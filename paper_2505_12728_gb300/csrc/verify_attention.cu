@@ -17,79 +17,42 @@
 //    one elected warp issues one TMA box per 16-token page and tensor
 //    (128-byte swizzle) straight from the block table, completing on an
 //    mbarrier; nothing else touches HBM in the loop.
-//  * All n_q * g query rows of a KV head share each K/V tile.  The rows are
+//  * All n_q * g query rows of a KV head share each K/V tile.  This kernel
+//    takes shapes with at most 16 such rows (MHA, n_q <= 16): the rows are
 //    the M dimension of bf16 m16n8k16 tensor-core MMAs (S = Q K^T and
 //    O += P V, fp32 accumulate); scores stay in registers, where an fp32
 //    online softmax (base 2, scale folded in) rescales the running output.
-//    With one row tile (MHA, n_q <= 16) the four warps split the tile's keys
-//    and combine in shared memory at the end of a piece.
+//    The four warps split each tile's keys and combine in shared memory at
+//    the end of a piece.  More rows per KV head (GQA) are a real dense
+//    contraction and go to the tcgen05 kernel in verify_attention_tc.cu.
 //  * A piece that covers a whole segment writes bf16 out and fp32 LSE
 //    directly.  Split segments are merged (deterministically, in piece
 //    order) in one of three ways:
 //      - cluster mode: for one sequence the grid is one thread-block cluster
 //        per KV head; the cluster's CTAs keep their partials in shared
 //        memory and merge them through distributed shared memory;
-//      - few rows (R <= 16): the CTA that takes the last ticket of the
-//        segment (an atomic counter; nobody waits) merges the fp32 partials;
-//      - many rows (GQA): verify_merge_kernel, a grid over rows and segments.
+//      - otherwise the CTA that takes the last ticket of the segment (an
+//        atomic counter; nobody waits) merges the fp32 partials;
+//      - the tcgen05 kernel's split segments (many rows): verify_merge_kernel,
+//        one thread per output quad.
 //  * Launches use programmatic stream serialisation: the partition, the
-//    block-table reads and the first copies run before griddepcontrol.wait,
-//    overlapping the previous kernel on the stream.
+//    block-table reads and the first copies of prefix tiles run before
+//    griddepcontrol.wait, overlapping the previous kernel on the stream
+//    (tiles holding draft positions are copied after it).
 //  * Page indices outside the pool and positions past a sequence's end are
 //    loaded as zero boxes (TMA out-of-bounds fill); bad indices set a bit in
 //    the status word.  Every mbarrier wait is bounded.
+#include <algorithm>
 #include <cmath>
 #include <map>
 #include <mutex>
 #include <tuple>
 
-#include "sf_device.cuh"
+#include "attn_common.cuh"
 #include "sf_host.h"
 
 namespace sf {
 
-constexpr int kTileTokens = 64;            // keys per ring stage
-constexpr int kPageTokens = SF_PAGE_SIZE;  // 16
-constexpr int kPagesPerTile = kTileTokens / kPageTokens;
-constexpr int kRowBytes = 128;             // one swizzled smem row (64 bf16)
-constexpr int kBeyondEnd = -2147483647 - 1;           // page past the sequence end
-
-struct AttnParams {
-  const __nv_bfloat16 *q;
-  const int32_t *block_table;
-  const int32_t *seq_lens;
-  __nv_bfloat16 *out;
-  float *lse;
-  uint32_t *status;
-  int2 *seg_desc;     // [B * H_kv]: {first CTA, pieces} of each segment
-  uint32_t *tickets;  // [B * H_kv], zero between calls (in-kernel merge)
-  int merge_in_kernel;  // 1: last CTA of a segment merges; 0: merge kernel
-  int cs;             // CTAs per cluster of the launch (1: no clusters)
-  int push;           // cluster mode: peers push partial rows into the merging CTA
-  int push_off;       // byte offset of the push area in dynamic shared memory
-  float *partials;    // [G + B * H_kv][R][D + 2]
-  int B, n_q, H_q, H_kv, group, R;
-  int num_pages, max_pages, max_tokens;
-  int oob_row;        // a tensor-map row beyond the pool: loads as zeros
-  float scale_log2;   // softmax_scale * log2(e)
-  int G;
-  int slot_stride;    // floats per partial slot: R*D (O) + R (max) + R (sum), padded to 4
-};
-
-// Floats per partial slot; a multiple of 4 so every slot starts 16-byte aligned.
-__host__ __device__ inline int partial_slot_floats(int R, int D) {
-  return (R * (D + 2) + 3) / 4 * 4;
-}
-
-// Shared-memory layout of one K or V tile (64 tokens): one TMA box per page,
-// [page][c / 8][token % 16][128 B], each 128-byte row 128B-swizzled.  Byte
-// offset of 16-byte chunk `c` (head_dim / 8 index) of token `t`:
-template <int D>
-__device__ __forceinline__ uint32_t swz(int t, int c) {
-  constexpr int kPageBytes = (D / 64) * kPageTokens * kRowBytes;
-  return static_cast<uint32_t>((t >> 4) * kPageBytes + (c >> 3) * (kPageTokens * kRowBytes) +
-                               (t & 15) * kRowBytes + (((c & 7) ^ (t & 7)) << 4));
-}
 
 template <int D, int STAGES, int NW>
 struct AttnSmem {
@@ -104,122 +67,9 @@ struct AttnSmem {
   static int bytes(int B) { return 1024 + kPrefixOffset + 4 * (2 * B + 2); }
 };
 
-// Exclusive prefix of per-sequence tile counts into s_prefix[0..B], clamped
-// sequence lengths into s_len[0..B-1].
-template <int NT>
-__device__ void tile_prefix(const AttnParams &p, int *s_prefix, int *s_len, int *s_warp) {
-  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  const int per = (p.B + NT - 1) / NT;
-  const int b0 = tid * per;
-  int local = 0;
-  for (int b = b0; b < b0 + per && b < p.B; ++b) {
-    int T = p.seq_lens[b];
-    if (T < p.n_q || T > p.max_tokens) {
-      set_status(p.status, SF_DEVICE_BAD_SEQLEN);
-      T = T < p.n_q ? p.n_q : p.max_tokens;
-    }
-    s_len[b] = T;
-    local += (T + kTileTokens - 1) / kTileTokens;
-  }
-  int incl = local;
-#pragma unroll
-  for (int o = 1; o < 32; o <<= 1) {
-    int v = __shfl_up_sync(0xffffffffu, incl, o);
-    if (lane >= o) incl += v;
-  }
-  if (lane == 31) s_warp[warp] = incl;
-  __syncthreads();
-  int warp_off = 0;
-  for (int w = 0; w < warp; ++w) warp_off += s_warp[w];
-  int run = warp_off + incl - local;
-  for (int b = b0; b < b0 + per && b < p.B; ++b) {
-    s_prefix[b] = run;
-    run += (s_len[b] + kTileTokens - 1) / kTileTokens;
-  }
-  if (tid == NT - 1) s_prefix[p.B] = warp_off + incl;
-}
 
-// The tile partition uses 32-bit arithmetic only (the host guarantees
-// fewer than 2^31 tiles and G <= 65535): CTA c owns the global tiles
-// [start(c), start(c+1)) with start(c) = floor(c * Tot / G), computed as
-// c*q + floor(c*r / G) with q = Tot / G, r = Tot % G (c*r < G^2 < 2^32).
-struct TilePartition {
-  uint32_t Tot, G, q, r;
-  __device__ __forceinline__ uint32_t start(uint32_t c) const { return c * q + (c * r) / G; }
-  // CTA whose range contains tile t: an fp32 estimate, then exact steps
-  __device__ __forceinline__ uint32_t owner(uint32_t t) const {
-    int c = static_cast<int>((static_cast<float>(t) + 0.5f) * (static_cast<float>(G) / static_cast<float>(Tot)));
-    c = c < 0 ? 0 : (c >= static_cast<int>(G) ? static_cast<int>(G) - 1 : c);
-    while (c > 0 && start(static_cast<uint32_t>(c)) > t) --c;
-    while (c + 1 < static_cast<int>(G) && start(static_cast<uint32_t>(c + 1)) <= t) ++c;
-    return static_cast<uint32_t>(c);
-  }
-};
-
-// Sequence b owning global tile t: H_kv * s_prefix[b] <= t < H_kv * s_prefix[b+1].
-__device__ __forceinline__ int find_sequence(uint32_t t, const int *s_prefix, int B, int H_kv) {
-  int lo = 0, hi = B - 1;
-  while (lo < hi) {
-    int mid = (lo + hi + 1) >> 1;
-    if (static_cast<uint32_t>(H_kv) * static_cast<uint32_t>(s_prefix[mid]) <= t) lo = mid; else hi = mid - 1;
-  }
-  return lo;
-}
-
-constexpr int kMergeBatch = 16;
-constexpr int kMaxGrid = 65535;  // CTAs of one launch (the partition uses 32-bit math)
 constexpr int kMaxCluster = 16;  // largest cluster launched (non-portable size)
 constexpr int kPushSlots = 2;    // rows a CTA merges in push mode (at most)
-
-template <bool kBypassL1, typename T>
-__device__ __forceinline__ T merge_load(const T *p) {
-  if constexpr (kBypassL1) return __ldcg(p);
-  else return *p;
-}
-
-// Combines the pieces of one output (row r, columns 4*c4 .. 4*c4+3) of a
-// split segment, in piece order:
-//   M = max_q m_q,  L = sum_q l_q 2^(m_q - M),  O = sum_q 2^(m_q - M) O_q / L.
-// The pieces are read in batches of kMergeBatch with an online rescale; all
-// loads of a batch are issued before any is used, so a batch costs one
-// memory round trip.  Partial slot layout: O [R][D], m [R], l [R].
-template <int D, bool kBypassL1>
-__device__ __forceinline__ void merge_one(const float *part0, size_t stride, int R, int r, int c4,
-                                          int n_pieces, float4 &o, float &M, float &Ls) {
-  const float *mrow = part0 + (size_t)R * D + r;
-  const float *lrow = mrow + R;
-  const float4 *orow = reinterpret_cast<const float4 *>(part0 + (size_t)r * D) + c4;
-  const size_t stride4 = stride / 4;
-  M = -INFINITY;
-  Ls = 0.f;
-  float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-  for (int q0 = 0; q0 < n_pieces; q0 += kMergeBatch) {
-    float mv[kMergeBatch], lv[kMergeBatch];
-    float4 xv[kMergeBatch];
-#pragma unroll
-    for (int u = 0; u < kMergeBatch; ++u) {
-      const bool in = q0 + u < n_pieces;
-      mv[u] = in ? merge_load<kBypassL1>(mrow + (q0 + u) * stride) : -INFINITY;
-      lv[u] = in ? merge_load<kBypassL1>(lrow + (q0 + u) * stride) : 0.f;
-      xv[u] = in ? merge_load<kBypassL1>(orow + (q0 + u) * stride4) : make_float4(0.f, 0.f, 0.f, 0.f);
-    }
-    float Mb = M;
-#pragma unroll
-    for (int u = 0; u < kMergeBatch; ++u) Mb = fmaxf(Mb, mv[u]);
-    const float a = exp2f(M - Mb);  // first batch: M = -inf, a = 0
-    Ls *= a;
-    acc.x *= a; acc.y *= a; acc.z *= a; acc.w *= a;
-#pragma unroll
-    for (int u = 0; u < kMergeBatch; ++u) {
-      const float w = exp2f(mv[u] - Mb);
-      Ls += lv[u] * w;
-      acc.x += xv[u].x * w; acc.y += xv[u].y * w; acc.z += xv[u].z * w; acc.w += xv[u].w * w;
-    }
-    M = Mb;
-  }
-  const float inv = 1.f / Ls;
-  o = make_float4(acc.x * inv, acc.y * inv, acc.z * inv, acc.w * inv);
-}
 
 template <int D, int KS, int NW, int STAGES>
 __global__ void __launch_bounds__(NW * 32, (NW == 4 ? 2 : 1))
@@ -348,21 +198,34 @@ verify_attention_kernel(const __grid_constant__ CUtensorMap tmap_k,
     const uint32_t piece_base = consumed;  // ring position of the piece's first tile
     int issued = prologue;                 // tiles of this piece issued so far
     int next_phys = 0;  // lanes 0..3 of warp 0: block-table entry of the next tile
-    if (warp == 0) {
-      if (lane < prologue) mbar_arrive_expect_tx(bar0 + 8 * ((piece_base + lane) % STAGES),
-                                                 L::kStageBytes);
-      __syncwarp();
-      if (lane < kPagesPerTile * prologue) {
-        const int j = lane / kPagesPerTile, pg = lane % kPagesPerTile;
-        issue((piece_base + j) % STAGES, pg, fetch_page(lt0 + j, pg));
+    // tiles j0 .. j1-1 of the prologue, one lane per page
+    auto issue_prologue = [&](int j0, int j1) {
+      if (warp == 0 && j1 > j0) {
+        if (lane >= j0 && lane < j1)
+          mbar_arrive_expect_tx(bar0 + 8 * ((piece_base + lane) % STAGES), L::kStageBytes);
+        __syncwarp();
+        if (lane < kPagesPerTile * (j1 - j0)) {
+          const int j = j0 + lane / kPagesPerTile, pg = lane % kPagesPerTile;
+          issue((piece_base + j) % STAGES, pg, fetch_page(lt0 + j, pg));
+        }
       }
-      if (lane < kPagesPerTile && prologue < n_tiles) next_phys = fetch_page(lt0 + prologue, lane);
+    };
+    // Before the wait on the previous kernel only tiles wholly inside the
+    // prefix are copied: the draft rows' K/V may be written by that kernel.
+    int pre = prologue;
+    if (!waited) {
+      pre = 0;
+      while (pre < prologue && (lt0 + pre + 1) * kTileTokens <= Lb) ++pre;
     }
+    issue_prologue(0, pre);
+    if (warp == 0 && lane < kPagesPerTile && prologue < n_tiles)
+      next_phys = fetch_page(lt0 + prologue, lane);
 
     if (!waited) {
       grid_dependency_wait();
       waited = true;
     }
+    issue_prologue(pre, prologue);
     if (lt0 == 0 && tid == 0) p.seg_desc[seg] = make_int2(c_first, aligned ? 1 : n_pieces);
     seg_b = b;
     seg_h = h_kv;
@@ -821,8 +684,8 @@ verify_attention_kernel(const __grid_constant__ CUtensorMap tmap_k,
 }
 
 // Merge for shapes with many rows per KV head (GQA): the pieces of every
-// split segment are combined by a grid over (row groups, segments), one
-// thread per 4 output columns of a row, in piece order (deterministic):
+// split segment are combined by a grid with one thread per 4 output columns
+// of a row (the whole output at once), in piece order (deterministic):
 //   M = max_q m_q,  L = sum_q l_q 2^(m_q - M),  O = sum_q 2^(m_q - M) O_q / L,
 //   lse = (M + log2 L) ln 2.
 // Pieces are read in batches of kMergeBatch with a running (online) rescale,
@@ -836,15 +699,16 @@ __global__ void __launch_bounds__(kMergeThreads)
 verify_merge_kernel(const __grid_constant__ AttnParams p) {
   constexpr float kLn2 = 0.6931471805599453f;
   constexpr int C4 = D / 4;                       // threads per row
-  constexpr int RPC = kMergeThreads / C4;         // rows per CTA
   grid_launch_dependents();
   grid_dependency_wait();
-  const int seg = blockIdx.y;
+  const long long item = (long long)blockIdx.x * kMergeThreads + threadIdx.x;
+  const int per_seg = p.R * C4;
+  if (item >= (long long)per_seg * p.B * p.H_kv) return;
+  const int seg = static_cast<int>(item / per_seg);
+  const int rem = static_cast<int>(item % per_seg);
+  const int r = rem / C4, c4 = rem % C4;
   const int2 desc = p.seg_desc[seg];              // {first CTA, pieces}
   if (desc.y <= 1) return;                        // the split kernel wrote it
-  const int r = blockIdx.x * RPC + threadIdx.x / C4;
-  const int c4 = threadIdx.x % C4;
-  if (r >= p.R) return;
   const size_t stride = (size_t)p.slot_stride;
   float4 ov;
   float M, Ls;
@@ -888,18 +752,11 @@ static AttnVariant make_variant() {
   return v;
 }
 
-static AttnVariant select_variant(int D, int R) {
-  const int rt = (R + 15) / 16;
-  if (D == 64) {
-    if (rt == 1) return make_variant<64, 4, 4>();
-    if (rt == 2) return make_variant<64, 2, 4>();
-    if (rt <= 4) return make_variant<64, 1, 4>();
-    return make_variant<64, 1, 8>();
-  }
-  if (rt == 1) return make_variant<128, 4, 4>();
-  if (rt == 2) return make_variant<128, 2, 4>();
-  if (rt <= 4) return make_variant<128, 1, 4>();
-  return make_variant<128, 1, 8>();
+// One row tile per KV head (R <= 16): the four warps split each tile's keys.
+// More rows go to the tcgen05 kernel (verify_attention_tc.cu).
+static AttnVariant select_variant(int D) {
+  if (D == 64) return make_variant<64, 4, 4>();
+  return make_variant<128, 4, 4>();
 }
 
 struct AttnLayout {
@@ -911,7 +768,7 @@ static AttnLayout attn_layout(int B, int H_kv, int R, int D, long long G) {
   const size_t segs = (size_t)B * H_kv;
   l.desc_off = 256;
   l.tickets_off = round_up(l.desc_off + 8 * segs, 256);
-  l.partials_off = round_up(l.tickets_off + 4 * segs, 256);
+  l.partials_off = round_up(l.tickets_off + 8 * segs, 256);
   l.total = round_up(l.partials_off + (size_t)(G + (long long)segs) * partial_slot_floats(R, D) * 4,
                      256);
   return l;
@@ -940,6 +797,7 @@ struct AttnPlan {
   int cs;        // CTAs per cluster (1: no clusters)
   int push;      // cluster mode pushes partial rows (few rows per merging CTA)
   int push_off;  // byte offset of the push area in shared memory
+  int tc;        // 1: the tcgen05 kernel (many rows per KV head)
 };
 
 // Largest dynamic shared memory a launch of variant v can ask for: the
@@ -1020,20 +878,37 @@ static int plan_attention(int B, int n_q, int H_q, int H_kv, int D, int max_page
   int st = current_device(&dev);
   if (st != SF_OK) return st;
   const int R = n_q * (H_q / H_kv);
-  plan->v = select_variant(D, R);
+  plan->v = select_variant(D);
   plan->smem = plan->v.smem_fixed + 8 * B;
   plan->push = 0;
   plan->push_off = 0;
+  plan->tc = 0;
+  const long long max_tiles =
+      (long long)B * H_kv * (((long long)max_pages_per_seq * SF_PAGE_SIZE + kTileTokens - 1) / kTileTokens);
+  if (max_tiles >= (1LL << 31))
+    return fail(SF_ERR_UNSUPPORTED, "B x H_kv x tiles per sequence = %lld tiles (limit 2^31)", max_tiles);
+  if (R > 16) {
+    // Many rows per KV head: a real dense contraction, run on the tcgen05
+    // tensor cores with one CTA per SM (the whole TMEM is one CTA's).
+    plan->tc = 1;
+    plan->cs = 1;
+    plan->smem = tc_smem_bytes(D, B);
+    if (tc_smem_bytes(D, SF_MAX_BATCH) > dev.max_smem_optin)
+      return fail(SF_ERR_UNSUPPORTED, "needs %d B shared memory, device allows %d",
+                  tc_smem_bytes(D, SF_MAX_BATCH), dev.max_smem_optin);
+    st = tc_setup(D, dev.ordinal);
+    if (st != SF_OK) return st;
+    long long G = num_splits > 0 && num_splits < dev.sm_count ? num_splits : dev.sm_count;
+    if (G > max_tiles) G = max_tiles;
+    plan->G = static_cast<int>(G < 1 ? 1 : G);
+    return SF_OK;
+  }
   if (max_dynamic_smem(plan->v) > dev.max_smem_optin)
     return fail(SF_ERR_UNSUPPORTED, "needs %d B shared memory, device allows %d",
                 max_dynamic_smem(plan->v), dev.max_smem_optin);
   int occ = 1;
   st = kernel_setup(plan->v, dev.ordinal, plan->smem, &occ);
   if (st != SF_OK) return st;
-  const long long max_tiles =
-      (long long)B * H_kv * (((long long)max_pages_per_seq * SF_PAGE_SIZE + kTileTokens - 1) / kTileTokens);
-  if (max_tiles >= (1LL << 31))
-    return fail(SF_ERR_UNSUPPORTED, "B x H_kv x tiles per sequence = %lld tiles (limit 2^31)", max_tiles);
   const long long capacity = (long long)dev.sm_count * occ;
   long long G = num_splits > 0 ? num_splits : capacity;
   plan->cs = 1;
@@ -1069,14 +944,17 @@ static int plan_attention(int B, int n_q, int H_q, int H_kv, int D, int max_page
   return SF_OK;
 }
 
-// TMA descriptors of the K and V caches, cached by (address, rows, head_dim)
-// so that repeated calls on the same caches skip the encoding.
-static int cache_tensor_map(CUtensorMap *out, const void *base, uint64_t rows, int head_dim) {
+// TMA descriptors of the K and V caches, cached by (address, rows,
+// head_dim, box) so that repeated calls on the same caches skip the encoding.
+// half_boxes = 0: one box brings a whole page (both 64-column halves when
+// head_dim is 128); 1: one box brings one 64-column half of a page.
+static int cache_tensor_map(CUtensorMap *out, const void *base, uint64_t rows, int head_dim,
+                            int half_boxes) {
   static std::mutex mu;
-  static std::map<std::tuple<const void *, uint64_t, int>, CUtensorMap> maps;
+  static std::map<std::tuple<const void *, uint64_t, int, int>, CUtensorMap> maps;
   {
     std::lock_guard<std::mutex> lock(mu);
-    auto it = maps.find({base, rows, head_dim});
+    auto it = maps.find({base, rows, head_dim, half_boxes});
     if (it != maps.end()) {
       *out = it->second;
       return SF_OK;
@@ -1085,11 +963,12 @@ static int cache_tensor_map(CUtensorMap *out, const void *base, uint64_t rows, i
   // head_dim 128: view each 256-byte token row as two 128-byte halves with
   // the halves outermost, {64 elements, rows, 2 halves} with byte strides
   // {256, 128}, so a {64, 16, 2} box brings a whole page in the shared
-  // layout [half][token][64].  head_dim 64: {64, rows}, box {64, 16}.
+  // layout [half][token][64] and a {64, 16, 1} box one half of a page.
+  // head_dim 64: {64, rows}, box {64, 16}.
   int st;
   if (head_dim == 128) {
     const uint64_t dims[3] = {64, rows, 2}, strides[2] = {256, 128};
-    const uint32_t box[3] = {64, SF_PAGE_SIZE, 2};
+    const uint32_t box[3] = {64, SF_PAGE_SIZE, half_boxes ? 1u : 2u};
     st = encode_tensor_map_bf16(out, base, 3, dims, strides, box);
   } else {
     const uint64_t dims[2] = {64, rows}, strides[1] = {128};
@@ -1099,7 +978,7 @@ static int cache_tensor_map(CUtensorMap *out, const void *base, uint64_t rows, i
   if (st != SF_OK) return st;
   std::lock_guard<std::mutex> lock(mu);
   if (maps.size() >= 4096) maps.clear();
-  maps.emplace(std::make_tuple(base, rows, head_dim), *out);
+  maps.emplace(std::make_tuple(base, rows, head_dim, half_boxes), *out);
   return SF_OK;
 }
 
@@ -1151,9 +1030,9 @@ int sf_verify_attention(const void *q, const void *k_cache, const void *v_cache,
 
   const uint64_t rows = (uint64_t)num_pages * H_kv * SF_PAGE_SIZE;
   CUtensorMap tk, tv;
-  st = cache_tensor_map(&tk, k_cache, rows, head_dim);
+  st = cache_tensor_map(&tk, k_cache, rows, head_dim, plan.tc);
   if (st != SF_OK) return st;
-  st = cache_tensor_map(&tv, v_cache, rows, head_dim);
+  st = cache_tensor_map(&tv, v_cache, rows, head_dim, 0);
   if (st != SF_OK) return st;
 
   AttnParams prm;
@@ -1206,11 +1085,17 @@ int sf_verify_attention(const void *q, const void *k_cache, const void *v_cache,
   cfg.stream = stream;
   cfg.attrs = attr;
   cfg.numAttrs = plan.cs > 1 ? 2 : 1;
-  cudaError_t e = cudaLaunchKernelEx(&cfg, plan.v.fn, tk, tv, prm);
-  if (e != cudaSuccess) return fail(SF_ERR_CUDA, "verify attention launch: %s", cudaGetErrorString(e));
+  cudaError_t e;
+  if (plan.tc) {
+    st = tc_launch(head_dim, plan.G, plan.smem, tk, tv, prm, stream);
+    if (st != SF_OK) return st;
+  } else {
+    e = cudaLaunchKernelEx(&cfg, plan.v.fn, tk, tv, prm);
+    if (e != cudaSuccess) return fail(SF_ERR_CUDA, "verify attention launch: %s", cudaGetErrorString(e));
+  }
   if (prm.merge_in_kernel) return SF_OK;
-  const int rpc = kMergeThreads / (head_dim / 4);
-  cfg.gridDim = dim3((R + rpc - 1) / rpc, B * H_kv);
+  const long long items = (long long)R * (head_dim / 4) * B * H_kv;
+  cfg.gridDim = dim3(static_cast<unsigned>((items + kMergeThreads - 1) / kMergeThreads));
   cfg.blockDim = dim3(kMergeThreads);
   cfg.dynamicSmemBytes = 0;
   cfg.numAttrs = 1;  // programmatic serialisation only, no clusters

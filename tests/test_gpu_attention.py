@@ -197,3 +197,22 @@ def test_uniform_segments_match_oracle(oracle_mod, B, n_q, H_q, H_kv, d, prefix)
     assert_attention_close(out, lse, ref_out, ref_lse)
     out2, lse2 = run_attention(case, num_splits=0)
     np.testing.assert_array_equal(out, out2)
+
+
+@pytest.mark.parametrize("n_q,H_q,H_kv", [(8, 28, 4), (3, 16, 2), (1, 8, 8)])
+def test_growing_scores_move_the_running_maximum(oracle_mod, n_q, H_q, H_kv):
+    # Scores that grow along the sequence (q all ones, every element of key t
+    # equal to t / 64) raise each row's maximum by about 16 (base 2) per
+    # 64-key tile, far beyond any lazy-rescale threshold, so the running
+    # output and sum are rescaled at every tile of every piece.
+    case = make_attention_case(2, n_q, H_q, H_kv, 128, [900, 1500], seed=95, spare_pages=2)
+    one = f32_to_bf16_bits(np.array([1.0], np.float32))[0]
+    case.q[...] = one
+    for b in range(2):
+        for t in range(int(case.seq_lens[b])):
+            page = case.block_table[0, b, t // 16]
+            case.k_cache[0, page, :, t % 16, :] = f32_to_bf16_bits(np.array([t / 64.0], np.float32))[0]
+    ref_out, ref_lse = oracle_attention(oracle_mod, case)
+    for splits in (0, 3):
+        out, lse = run_attention(case, num_splits=splits)
+        assert_attention_close(out, lse, ref_out, ref_lse)
