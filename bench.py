@@ -145,6 +145,27 @@ def accept_bytes(wl, mode_sampling_rows: int) -> int:
     return wl.B * (wl.k + 1) * wl.V * 4 + mode_sampling_rows * wl.V * 4 * 2
 
 
+# Sources whose code (comments and layout removed) a committed ncu summary
+# was taken on, per attention kernel, and the summary of each workload.
+KERNEL_SOURCES = {
+    "verify_attention_kernel": ["paper_2505_12728_gb300/csrc/verify_attention.cu",
+                                "paper_2505_12728_gb300/csrc/attn_common.cuh",
+                                "paper_2505_12728_gb300/csrc/sf_device.cuh"],
+    "verify_attention_tc_kernel": ["paper_2505_12728_gb300/csrc/verify_attention_tc.cu",
+                                   "paper_2505_12728_gb300/csrc/attn_common.cuh",
+                                   "paper_2505_12728_gb300/csrc/sf_device.cuh"],
+}
+PROFILES = {"image7b": "profiles/verify_attention_image7b.md",
+            "video": "profiles/verify_attention_tc_video.md"}
+
+
+def attention_kernel(wl):
+    """The kernel the library runs for a workload: the tcgen05 kernel when a
+    KV head has more than 16 query rows, else the mma.sync kernel."""
+    return "verify_attention_tc_kernel" if wl.rows * (wl.H_q // wl.H_kv) > 16 \
+        else "verify_attention_kernel"
+
+
 def profiled_traffic(kernel_sources, profile):
     """DRAM bytes per launch from a committed ncu summary, or None when the
     kernel's sources changed since the counters were taken."""
@@ -449,6 +470,7 @@ def run_ours(args):
     acc_launch_ms = sum(acc_ms) / args.steps
     status = sfv.read_device_status(ws_att) | sfv.read_device_status(ws_acc)
 
+    kernel = attention_kernel(wl)
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True,
@@ -463,20 +485,19 @@ def run_ours(args):
         "mean_accepted": float(n_acc.float().mean().item()),
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                      "frac": achieved / peak,
-                     "traffic": (profiled_traffic(
-                         ["paper_2505_12728_gb300/csrc/verify_attention.cu",
-                          "paper_2505_12728_gb300/csrc/sf_device.cuh"],
-                         "profiles/verify_attention_image7b.md")
-                         if wl.name == "image7b" else None),
+                     "traffic": (profiled_traffic(KERNEL_SOURCES[kernel], PROFILES[wl.name])
+                                 if wl.name in PROFILES else None),
                      "algorithmic_bytes": bytes_layer,
-                     "kernel": "verify_attention_kernel",
+                     "kernel": kernel,
                      "peak_source": f"{peak_kind} copy bandwidth (MEASURED_PEAKS.json hbm_gbs)"},
         "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d,
                 "d2h_bytes_per_step": d2h, "ms_per_step": e2e_ms / args.steps,
                 "host_result_matches_device": h_ok},
         "launch": "cuda_graph" if use_graph else "eager",
         "eager_ms_per_step": eager_ms,
-        "gpu_launches": args.steps * (L * (1 if wl.rows <= 16 else 2) + 2),
+        # per step: each layer's attention kernel (+ the merge kernel after the
+        # tcgen05 kernel), then the two acceptance kernels
+        "gpu_launches": args.steps * (L * (2 if kernel == "verify_attention_tc_kernel" else 1) + 2),
         "clocks": clk,
         "device_status": status,
     }
