@@ -254,7 +254,7 @@ def run_reference(args):
                                                   workload)
     from oracle import oracle
     oracle.build()
-    wl = workload(args.workload)
+    wl = workload(args.workload, **({"layers": args.layers} if args.layers else {}))
     att = make_attention_inputs(wl, layers=min(wl.layers, 2))
     acc = make_accept_inputs(wl)
     for w in range(args.warmup):
@@ -308,7 +308,7 @@ def run_ours(args):
                                                   workload)
     build_lib.build()
     sfv.load_library()
-    wl = workload(args.workload)
+    wl = workload(args.workload, **({"layers": args.layers} if args.layers else {}))
     att = make_attention_inputs(wl)
     acc = make_accept_inputs(wl)
 
@@ -517,6 +517,8 @@ def main(argv=None):
     ap.add_argument("--warmup", type=int, default=50)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", default="image7b")
+    ap.add_argument("--layers", type=int, default=0,
+                    help="independent attention layers per step (default: the workload's)")
     ap.add_argument("--cpu-budget", type=float, default=12.0,
                     help="seconds of oracle work for the cpu_baseline sample")
     ap.add_argument("--no-cpu-baseline", action="store_true")

@@ -1,7 +1,8 @@
 // accept.cu -- fused speculative acceptance for sm_103a.
 //
-// The verification rule (Sec. 3.1; Sec. 3.3 "the standard token-wise
-// acceptance-rejection rule"): with p_i = softmax(target_logits_i / tau) and
+// The verification rule (Sec. 3.1; Sec. 3.3 names it the usual token-by-token
+// accept/reject rule of speculative sampling): with
+// p_i = softmax(target_logits_i / tau) and
 // the draft distribution q_i, draft T'_{i+1} = x_i is accepted iff
 // u_i * q_i(x_i) < p_i(x_i) (probability min(1, p/q)); decisions are taken in
 // order up to the first rejection j; the token at position j is drawn by
@@ -18,13 +19,13 @@
 //    registers; the CTA whose chunk holds the row's draft token also records
 //    that token's logit and draft probability.  The last CTA of a sequence
 //    to finish (one atomic ticket; nobody waits) combines every row, one warp
-//    per row, in fp64, and takes the k accept/reject decisions in fp64.
+//    per row, and takes the k accept/reject decisions (float-float, below).
 //  * accept_draw_kernel, grid (chunks, B), launched with programmatic stream
 //    serialisation so that it is resident while the first kernel drains: for
 //    sampled sequences each CTA sums the residual (or bonus) mass of a chunk
 //    of row j; the last CTA of the sequence locates the chunk holding u_k * S
-//    with an fp64 scan over chunk sums and scans that chunk in ascending
-//    token order.
+//    with a float-float scan over chunk sums and scans that chunk in
+//    ascending token order.
 // Arithmetic: per-element terms are fp32 (expf, explicitly rounded products
 // and differences, identical wherever a value is recomputed); sums, scans and
 // the accept tests use float-float numbers (an unevaluated sum hi + lo of two
@@ -537,7 +538,7 @@ accept_draw_kernel(const __grid_constant__ AccParams p) {
   }
   const ff target = ff_mul(total, u_k);
 
-  // chunk holding the target: inclusive fp64 scan over chunk sums in order;
+  // chunk holding the target: inclusive float-float scan over chunk sums in order;
   // chunk cc covers [excl, incl), and excl of cc is bit-identical to incl of
   // cc - 1, so the intervals tile [0, total) without gaps or overlaps
   if (tid == 0) { s_chunk = INT_MAX; s_base = ff_of(0.f); }
