@@ -72,6 +72,8 @@ def _load():
         lib.oracle_argmax.restype = I
         lib.oracle_accept.argtypes = [P, P, P, P, P, I, I, I, P, P, P, P]
         lib.oracle_accept.restype = I
+        lib.oracle_kv_commit.argtypes = [P, P, P, P, P, I, I, I, I, I, I]
+        lib.oracle_kv_commit.restype = I
         _lib = lib
         return lib
 
@@ -185,3 +187,32 @@ def accept(target_logits, draft_probs, draft_tokens, uniforms, temperature):
         raise OracleError(f"oracle_accept status {st}")
     return dict(num_accepted=num_accepted, out_tokens=out_tokens, accept_ratio=ratio,
                 margin=margin)
+
+
+ORACLE_ERR_PAGES = 5
+
+
+def kv_commit(seq_lens, block_table, free_pages, free_count, num_accepted, n_q, n_q_next,
+              page_size=16):
+    """Cache bookkeeping after acceptance (Sec. 3.1, Sec. 3.3): keep the first
+    min(a + 1, n_q) verified rows of each sequence, set seq_lens for the next
+    n_q_next rows and map exactly their pages through the free-page stack.
+
+    seq_lens [B] int32, block_table [B][max_pages] int32, free_pages
+    [capacity] int32 (entries [0, free_count) are free pages), num_accepted
+    [B] int32.  Inputs are not modified.  Returns (status, seq_lens,
+    block_table, free_pages, free_count); status is ORACLE_OK,
+    ORACLE_ERR_ARG or ORACLE_ERR_PAGES, and on an error the returned arrays
+    equal the inputs.
+    """
+    lib = _load()
+    sl = np.array(seq_lens, dtype=np.int32, copy=True, order="C")
+    bt = np.array(block_table, dtype=np.int32, copy=True, order="C")
+    fp = np.array(free_pages, dtype=np.int32, copy=True, order="C")
+    fc = np.array([int(free_count)], dtype=np.int32)
+    na = _c(num_accepted, np.int32)
+    B, max_pages = bt.shape
+    assert sl.shape == (B,) and na.shape == (B,)
+    st = lib.oracle_kv_commit(_ptr(sl), _ptr(bt), _ptr(fp), _ptr(fc), _ptr(na), B, n_q, n_q_next,
+                              max_pages, page_size, fp.shape[0])
+    return int(st), sl, bt, fp, int(fc[0])

@@ -402,3 +402,94 @@ int oracle_accept(const float *target_logits, const float *draft_probs,
     free(r);
     return ORACLE_OK;
 }
+
+/*
+ * 4. KV commit after acceptance (Sec. 3.1: the accepted candidates join the
+ *    context and generation continues from the first rejected position;
+ *    Sec. 3.3: the next draft block starts from the emitted token).
+ *
+ *    Reading adopted (the paper gives no cache mechanics): the n_q rows
+ *    verified for sequence b sit at cache positions L_b .. L_b + n_q - 1,
+ *    L_b = seq_lens[b] - n_q, and row i belongs to the i-th token of the
+ *    verified block, whose first token is the previously emitted one.  With
+ *    a = num_accepted[b] drafts accepted, the first keep = min(a + 1, n_q)
+ *    rows stay valid and the rest are dropped: the cached length becomes
+ *    L'_b = L_b + keep.  The next verification of n_q_next rows writes them
+ *    at L'_b .., so seq_lens[b] becomes L'_b + n_q_next, and the block table
+ *    must map exactly need_b = ceil(seq_lens[b] / page_size) logical pages
+ *    (it mapped ceil(old seq_lens[b] / page_size) before).
+ *
+ *    Page bookkeeping through a stack of free physical pages
+ *    free_pages[0 .. *free_count):
+ *      1. for b = 0 .. B-1, for each logical page lp = need_b .. had_b - 1
+ *         (ascending): push block_table[b][lp] and set the entry to -1;
+ *      2. then for b = 0 .. B-1, for each logical page lp = had_b ..
+ *         need_b - 1 (ascending): take the stack entry at index
+ *         (top after step 1) - (total pages taken) + (count taken so far),
+ *         i.e. the taken pages are the topmost entries, assigned bottom-up;
+ *      3. the stack keeps its entries below that point.
+ *    All or nothing: if any sequence is invalid (seq_lens[b] < n_q,
+ *    num_accepted[b] < 0, need_b > max_pages) the result is
+ *    ORACLE_ERR_ARG, and if the stack would overflow `capacity` or run out
+ *    of pages it is ORACLE_ERR_PAGES; in both cases nothing is modified.
+ */
+#define ORACLE_ERR_PAGES 5
+
+/* Cached length for the next step and logical pages before / after. */
+static void commit_plan(int T, int a, int n_q, int n_q_next, int page_size, long long *next_len,
+                        long long *had, long long *need)
+{
+    const int keep = a + 1 < n_q ? a + 1 : n_q;
+    *next_len = (long long)(T - n_q) + keep + n_q_next;
+    *had = ((long long)T + page_size - 1) / page_size;
+    *need = (*next_len + page_size - 1) / page_size;
+}
+
+int oracle_kv_commit(int32_t *seq_lens, int32_t *block_table, int32_t *free_pages,
+                     int32_t *free_count, const int32_t *num_accepted, int B, int n_q,
+                     int n_q_next, int max_pages, int page_size, int capacity)
+{
+    if (B < 1 || n_q < 1 || n_q_next < 1 || max_pages < 1 || page_size < 1 || capacity < 0 ||
+        *free_count < 0 || *free_count > capacity)
+        return ORACLE_ERR_ARG;
+    long long pushed = 0, taken = 0, next_len, had, need;
+    for (int b = 0; b < B; ++b) {
+        if (seq_lens[b] < n_q || num_accepted[b] < 0)
+            return ORACLE_ERR_ARG;
+        commit_plan(seq_lens[b], num_accepted[b], n_q, n_q_next, page_size, &next_len, &had,
+                    &need);
+        if (need > max_pages || had > max_pages)
+            return ORACLE_ERR_ARG;
+        if (need < had)
+            pushed += had - need;
+        else
+            taken += need - had;
+    }
+    const long long top = (long long)*free_count + pushed;
+    if (top > capacity || taken > top)
+        return ORACLE_ERR_PAGES;
+
+    /* step 1: surplus pages onto the stack, in sequence order */
+    long long sp = *free_count;
+    for (int b = 0; b < B; ++b) {
+        commit_plan(seq_lens[b], num_accepted[b], n_q, n_q_next, page_size, &next_len, &had,
+                    &need);
+        int32_t *row = block_table + (size_t)b * max_pages;
+        for (long long lp = need; lp < had; ++lp) {
+            free_pages[sp++] = row[lp];
+            row[lp] = -1;
+        }
+    }
+    /* step 2: missing pages from the top `taken` stack entries, bottom-up */
+    long long take = top - taken;
+    for (int b = 0; b < B; ++b) {
+        commit_plan(seq_lens[b], num_accepted[b], n_q, n_q_next, page_size, &next_len, &had,
+                    &need);
+        int32_t *row = block_table + (size_t)b * max_pages;
+        for (long long lp = had; lp < need; ++lp)
+            row[lp] = free_pages[take++];
+        seq_lens[b] = (int32_t)next_len;
+    }
+    *free_count = (int32_t)(top - taken);
+    return ORACLE_OK;
+}

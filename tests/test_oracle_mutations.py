@@ -41,6 +41,16 @@ MUTANTS = {
     "slot_shifted": ("int slot = t % page_size;", "int slot = (t + 1) % page_size;"),
     "values_read_from_keys": ("        const uint16_t *vrow =\n            v_cache +",
                               "        const uint16_t *vrow =\n            k_cache +"),
+    "commit_keeps_accepted_rows_only": ("const int keep = a + 1 < n_q ? a + 1 : n_q;",
+                                        "const int keep = a < n_q ? a : n_q;"),
+    "commit_forgets_next_rows": ("*next_len = (long long)(T - n_q) + keep + n_q_next;",
+                                 "*next_len = (long long)(T - n_q) + keep;"),
+    "commit_takes_top_down": ("            row[lp] = free_pages[take++];",
+                              "            row[lp] = free_pages[top - 1 - (take++ - (top - taken))];"),
+    "commit_pushes_descending": ("        for (long long lp = need; lp < had; ++lp) {\n            free_pages[sp++] = row[lp];",
+                                 "        for (long long lp = need; lp < had; ++lp) {\n            free_pages[sp++] = row[had - 1 - (lp - need)];"),
+    "commit_page_count_floor": ("*need = (*next_len + page_size - 1) / page_size;",
+                                "*need = *next_len / page_size;"),
 }
 
 
@@ -67,6 +77,7 @@ def test_pins_reject_mutant(name, source, tmp_path):
     proc = subprocess.run(
         [sys.executable, "-m", "pytest", "-x", "-q", "-p", "no:cacheprovider",
          os.path.join(ROOT, "tests", "test_oracle_attention.py"),
-         os.path.join(ROOT, "tests", "test_oracle_accept.py")],
+         os.path.join(ROOT, "tests", "test_oracle_accept.py"),
+         os.path.join(ROOT, "tests", "test_oracle_kv_commit.py")],
         cwd=ROOT, env=env, capture_output=True, text=True, timeout=600)
     assert proc.returncode != 0, f"mutant {name} survived the oracle pins:\n{proc.stdout[-2000:]}"
