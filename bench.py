@@ -418,6 +418,32 @@ def run_ours(args):
     tokens = wl.B * wl.k * world * args.steps
     value = tokens / (total_ms / 1e3)
 
+    # ---- KV commit after acceptance (outside the step: it changes the cache
+    # state).  Timed in a steady state on a copy of layer 0's table: a = 0
+    # keeps one verified row and the next step verifies n_q - 1 rows, so every
+    # length and page stays put; 100 commits replayed as one graph.
+    commit_us = None
+    if wl.rows >= 2:
+        c_sl, c_bt = sl.clone(), bt[0].clone()
+        c_fp = torch.zeros(16, dtype=torch.int32, device=dev)
+        c_fc = torch.zeros(1, dtype=torch.int32, device=dev)
+        c_acc = torch.zeros(wl.B, dtype=torch.int32, device=dev)
+        c_ws = sfv.new_workspace(sfv.kv_commit_workspace_size(), dev)
+        commit_once = lambda: sfv.kv_commit(c_sl, c_bt, c_fp, c_fc, c_acc, wl.rows, wl.rows - 1,
+                                            workspace=c_ws, stream=stream)
+        commit_once()
+        g_com = capture(lambda: [commit_once() for _ in range(100)])
+        g_com.replay()
+        c0 = torch.cuda.Event(enable_timing=True)
+        c1 = torch.cuda.Event(enable_timing=True)
+        c0.record(stream)
+        for _ in range(5):
+            g_com.replay()
+        c1.record(stream)
+        torch.cuda.synchronize()
+        commit_us = c0.elapsed_time(c1) * 1e3 / 500
+        assert sfv.read_device_status(c_ws) == 0 and torch.equal(c_sl, sl)
+
     # ---- end to end through host buffers ----
     pin = lambda a: torch.from_numpy(np.ascontiguousarray(a)).pin_memory()
     h_q = pin(att.q.view(np.int16))
@@ -482,6 +508,7 @@ def run_ours(args):
         "kv_gbs": achieved,
         "kv_frac_of_nominal_8tbs": achieved / NOMINAL_HBM_GBS,
         "accept_gbs": accept_bytes(wl, sampling_rows) / (acc_launch_ms / 1e3) / 1e9,
+        "kv_commit_us": commit_us,
         "mean_accepted": float(n_acc.float().mean().item()),
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                      "frac": achieved / peak,

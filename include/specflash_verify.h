@@ -67,6 +67,7 @@ typedef enum {
 #define SF_DEVICE_BAD_TOKEN 0x2u /* draft token outside [0, V)                */
 #define SF_DEVICE_TIMEOUT 0x4u   /* a bounded wait on a copy gave up (~1 s)   */
 #define SF_DEVICE_BAD_SEQLEN 0x8u /* seq_lens[b] outside [n_q, max_pages*16]   */
+#define SF_DEVICE_OUT_OF_PAGES 0x10u /* sf_kv_commit: free-page stack too small */
 
 /* Limits of this build. */
 #define SF_PAGE_SIZE 16      /* tokens per KV page                            */
@@ -197,6 +198,53 @@ int sf_accept(const float *target_logits, const float *draft_probs,
               int B, int k, int V, int32_t *num_accepted, int32_t *out_tokens,
               float *accept_ratio, void *workspace, size_t workspace_bytes,
               cudaStream_t stream);
+
+/* ------------------------------------------------------------------------ */
+/* KV commit after acceptance (Sec. 3.1: the accepted candidates join the    */
+/* context and decoding continues from the first rejected position; Sec.    */
+/* 3.3: the next draft block starts from the emitted token).  The paper      */
+/* gives no cache mechanics; this call keeps a paged cache consistent on the */
+/* device, with no host round trip, between two verification steps.         */
+/*                                                                           */
+/* For each sequence b, with a = num_accepted[b] (from sf_accept): of the    */
+/* n_q rows verified at cache positions L_b .. L_b + n_q - 1                 */
+/* (L_b = seq_lens[b] - n_q), the first keep = min(a + 1, n_q) stay -- row i */
+/* holds the i-th token of the verified block, whose first token is the one  */
+/* emitted by the previous step -- and the rest are dropped.  The next step  */
+/* verifies n_q_next rows written at L_b + keep ..:                           */
+/*   seq_lens[b] <- L_b + keep + n_q_next,                                   */
+/* and the block table maps exactly need_b = ceil(seq_lens[b] / 16) logical  */
+/* pages (it mapped ceil(old seq_lens[b] / 16) before):                      */
+/*   1. pages no longer needed are pushed onto the free-page stack, in       */
+/*      sequence order and ascending logical page, and their entries set to  */
+/*      -1;                                                                  */
+/*   2. missing pages are then taken from the topmost stack entries, assigned */
+/*      bottom-up in sequence order and ascending logical page.              */
+/* Deterministic; all or nothing: if any seq_lens[b] < n_q, num_accepted[b]  */
+/* < 0 or need_b > max_pages_per_seq, SF_DEVICE_BAD_SEQLEN is set, and if the */
+/* stack would run out of pages or overflow `capacity`,                      */
+/* SF_DEVICE_OUT_OF_PAGES is set; in both cases nothing is modified.         */
+/*                                                                           */
+/* seq_lens      int32 [B], in/out.                                          */
+/* block_table   int32 [B][max_pages_per_seq], in/out.                       */
+/* free_pages    int32 [capacity], in/out: entries [0, *free_count) are free  */
+/*               physical page ids (a stack, top at the end).                */
+/* free_count    int32 [1], in/out (device memory).                          */
+/* num_accepted  int32 [B] in [0, k].                                        */
+/* B <= 1024; 1 <= n_q, n_q_next <= 16; page_size 16.                        */
+/* workspace     >= sf_kv_commit_workspace_size() bytes, 256-byte aligned,   */
+/*               zero-filled before first use (status word).                 */
+/* The next sf_verify_attention reads seq_lens and the block table before    */
+/* waiting for the kernel that precedes it on the stream, so that kernel must */
+/* not be this one (in a decoding loop the K/V append of the next draft rows */
+/* comes in between).                                                        */
+/* ------------------------------------------------------------------------ */
+size_t sf_kv_commit_workspace_size(void);
+
+int sf_kv_commit(int32_t *seq_lens, int32_t *block_table, int32_t *free_pages,
+                 int32_t *free_count, const int32_t *num_accepted, int B, int n_q, int n_q_next,
+                 int max_pages_per_seq, int page_size, int capacity, void *workspace,
+                 size_t workspace_bytes, cudaStream_t stream);
 
 #ifdef __cplusplus
 }

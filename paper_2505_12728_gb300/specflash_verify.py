@@ -22,6 +22,7 @@ SF_DEVICE_BAD_PAGE = 0x1
 SF_DEVICE_BAD_TOKEN = 0x2
 SF_DEVICE_TIMEOUT = 0x4
 SF_DEVICE_BAD_SEQLEN = 0x8
+SF_DEVICE_OUT_OF_PAGES = 0x10
 PAGE_SIZE = 16
 
 EXPORTED_SYMBOLS = (
@@ -29,6 +30,7 @@ EXPORTED_SYMBOLS = (
     "sf_read_device_status", "sf_verify_attention_workspace_size", "sf_verify_attention",
     "sf_verify_attention_noalloc",
     "sf_accept_workspace_size", "sf_accept",
+    "sf_kv_commit_workspace_size", "sf_kv_commit",
 )
 
 _lock = threading.Lock()
@@ -81,6 +83,10 @@ def load_library(path: str | None = None):
         lib.sf_accept_workspace_size.restype = S
         lib.sf_accept.argtypes = [P, P, P, P, P, I, I, I, P, P, P, P, S, P]
         lib.sf_accept.restype = I
+        lib.sf_kv_commit_workspace_size.argtypes = []
+        lib.sf_kv_commit_workspace_size.restype = S
+        lib.sf_kv_commit.argtypes = [P, P, P, P, P, I, I, I, I, I, I, P, S, P]
+        lib.sf_kv_commit.restype = I
         _lib = lib
         return lib
 
@@ -250,3 +256,28 @@ def accept(target_logits, draft_probs, draft_tokens, uniforms, temperature, *,
         _ptr(temperature), B, k, V, _ptr(num_accepted), _ptr(out_tokens), _ptr(accept_ratio),
         _ptr(workspace), workspace.numel(), _stream_handle(stream)))
     return num_accepted, out_tokens, accept_ratio
+
+
+def kv_commit_workspace_size() -> int:
+    return int(load_library().sf_kv_commit_workspace_size())
+
+
+def kv_commit(seq_lens, block_table, free_pages, free_count, num_accepted, n_q, n_q_next, *,
+              workspace=None, stream=None):
+    """sf_kv_commit, in place: seq_lens int32 [B], block_table int32
+    [B][max_pages], free_pages int32 [capacity] (a stack of free page ids),
+    free_count int32 [1], num_accepted int32 [B] (from accept).  Keeps the
+    first min(a + 1, n_q) verified rows of each sequence, prepares seq_lens
+    for the next n_q_next rows and maps exactly their pages."""
+    B, max_pages = block_table.shape
+    _need(seq_lens, "seq_lens", torch.int32, (B,))
+    _need(block_table, "block_table", torch.int32)
+    _need(free_pages, "free_pages", torch.int32)
+    _need(free_count, "free_count", torch.int32, (1,))
+    _need(num_accepted, "num_accepted", torch.int32, (B,))
+    if workspace is None:
+        workspace = new_workspace(kv_commit_workspace_size(), seq_lens.device)
+    _check(load_library().sf_kv_commit(
+        _ptr(seq_lens), _ptr(block_table), _ptr(free_pages), _ptr(free_count), _ptr(num_accepted),
+        B, n_q, n_q_next, max_pages, PAGE_SIZE, free_pages.numel(), _ptr(workspace),
+        workspace.numel(), _stream_handle(stream)))
