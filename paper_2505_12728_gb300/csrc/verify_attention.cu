@@ -69,6 +69,7 @@ struct AttnSmem {
 
 
 constexpr int kMaxCluster = 16;  // largest cluster launched (non-portable size)
+constexpr int kPrefetchLines = 64;  // block-table lines prefetched for one sequence
 constexpr int kPushSlots = 2;    // rows a CTA merges in push mode (at most)
 
 template <int D, int KS, int NW, int STAGES>
@@ -106,6 +107,10 @@ verify_attention_kernel(const __grid_constant__ CUtensorMap tmap_k,
   // first K/V copies) runs before grid_dependency_wait(); Q is read and
   // results are written only after it.
   grid_launch_dependents();
+  // one sequence: bring its block-table row toward the SM while seq_lens is
+  // read (the row is needed as soon as the partition is known)
+  if (p.B == 1 && tid < kPrefetchLines && tid * 32 < p.max_pages)
+    prefetch_l2(p.block_table + tid * 32);
   if (tid == 0) {
     for (int s = 0; s < STAGES; ++s) mbar_init(bar0 + 8 * s, 1);
     fence_mbar_init();
@@ -133,7 +138,12 @@ verify_attention_kernel(const __grid_constant__ CUtensorMap tmap_k,
   // through global memory.  Decided per cluster (identically by its CTAs);
   // every CTA of an aligned cluster has exactly one piece.
   bool aligned = false;
-  if (p.cs > 1 && G == p.G) {
+  // one sequence: its H_kv segments have equal length, so with G = H_kv x cs
+  // every cluster is exactly one segment (no partition arithmetic needed)
+  const bool one_seq_clusters = p.cs > 1 && p.B == 1 && G == p.G && G == p.H_kv * p.cs;
+  if (one_seq_clusters) {
+    aligned = true;
+  } else if (p.cs > 1 && G == p.G) {
     const uint32_t k = blockIdx.x / p.cs;
     const uint32_t c0 = part_of.start(k * p.cs), c1 = part_of.start((k + 1) * p.cs);
     const int bb = find_sequence(c0, s_prefix, p.B, p.H_kv);
@@ -150,18 +160,30 @@ verify_attention_kernel(const __grid_constant__ CUtensorMap tmap_k,
 
   for (uint32_t t = t_begin; t < t_end && !timed_out;) {
     // ---- locate the piece: segment (b, h_kv), local tiles [lt0, lt1) ----
-    const int b = find_sequence(t, s_prefix, p.B, p.H_kv);
-    const int tiles_b = s_prefix[b + 1] - s_prefix[b];
-    const uint32_t seg_base = static_cast<uint32_t>(p.H_kv) * static_cast<uint32_t>(s_prefix[b]);
-    const int h_kv = static_cast<int>((t - seg_base) / static_cast<uint32_t>(tiles_b));
-    const int lt0 = static_cast<int>((t - seg_base) % static_cast<uint32_t>(tiles_b));
-    const uint32_t left = t_end - t;
-    const int n_tiles = left < static_cast<uint32_t>(tiles_b - lt0) ? static_cast<int>(left) : tiles_b - lt0;
-    const uint32_t seg_first = seg_base + static_cast<uint32_t>(h_kv) * static_cast<uint32_t>(tiles_b);
+    int b, tiles_b, h_kv, lt0, n_tiles, c_first, n_pieces;
+    if (one_seq_clusters) {
+      // cluster k = KV head k; CTA rank r holds tiles [r tiles / cs, (r+1) tiles / cs)
+      b = 0;
+      tiles_b = s_prefix[1];
+      h_kv = static_cast<int>(blockIdx.x) / p.cs;
+      const int rank = static_cast<int>(blockIdx.x) - h_kv * p.cs;
+      lt0 = rank * tiles_b / p.cs;
+      n_tiles = (rank + 1) * tiles_b / p.cs - lt0;
+      c_first = h_kv * p.cs;
+      n_pieces = p.cs;
+    } else {
+      b = find_sequence(t, s_prefix, p.B, p.H_kv);
+      tiles_b = s_prefix[b + 1] - s_prefix[b];
+      const uint32_t seg_base = static_cast<uint32_t>(p.H_kv) * static_cast<uint32_t>(s_prefix[b]);
+      h_kv = static_cast<int>((t - seg_base) / static_cast<uint32_t>(tiles_b));
+      lt0 = static_cast<int>((t - seg_base) % static_cast<uint32_t>(tiles_b));
+      const uint32_t left = t_end - t;
+      n_tiles = left < static_cast<uint32_t>(tiles_b - lt0) ? static_cast<int>(left) : tiles_b - lt0;
+      const uint32_t seg_first = seg_base + static_cast<uint32_t>(h_kv) * static_cast<uint32_t>(tiles_b);
+      c_first = static_cast<int>(part_of.owner(seg_first));
+      n_pieces = static_cast<int>(part_of.owner(seg_first + tiles_b - 1)) - c_first + 1;
+    }
     const int seg = b * p.H_kv + h_kv;
-    const int c_first = static_cast<int>(part_of.owner(seg_first));
-    const int c_last = static_cast<int>(part_of.owner(seg_first + tiles_b - 1));
-    const int n_pieces = c_last - c_first + 1;
     const int T = s_len[b];
     const int Lb = T - p.n_q;
     t += n_tiles;
