@@ -74,6 +74,8 @@ def _load():
         lib.oracle_accept.restype = I
         lib.oracle_kv_commit.argtypes = [P, P, P, P, P, I, I, I, I, I, I]
         lib.oracle_kv_commit.restype = I
+        lib.oracle_sample.argtypes = [P, P, P, I, I, P, P, P]
+        lib.oracle_sample.restype = I
         _lib = lib
         return lib
 
@@ -216,3 +218,40 @@ def kv_commit(seq_lens, block_table, free_pages, free_count, num_accepted, n_q, 
     st = lib.oracle_kv_commit(_ptr(sl), _ptr(bt), _ptr(fp), _ptr(fc), _ptr(na), B, n_q, n_q_next,
                               max_pages, page_size, fp.shape[0])
     return int(st), sl, bt, fp, int(fc[0])
+
+
+def sample(logits, uniforms, temperature):
+    """Draft-tail sampling (Algorithm 1): P' = softmax(logits / tau) per row,
+    T' by inverse CDF with the row's uniform (ascending token id, strict <);
+    tau <= 0: first argmax, one-hot P'.  logits [R][V] fp32, uniforms [R]
+    fp32, temperature [R] fp32.  Returns (probs [R][V] float64, tokens [R]
+    int32, margin [R] float64: distance of each draw to the nearest CDF
+    boundary)."""
+    lib = _load()
+    logits = _c(logits, np.float32)
+    uniforms = _c(uniforms, np.float32)
+    temperature = _c(temperature, np.float32)
+    R, V = logits.shape
+    assert uniforms.shape == (R,) and temperature.shape == (R,)
+    probs = np.zeros((R, V), np.float64)
+    tokens = np.zeros(R, np.int32)
+    margin = np.zeros(R, np.float64)
+    st = lib.oracle_sample(_ptr(logits), _ptr(uniforms), _ptr(temperature), R, V, _ptr(probs),
+                           _ptr(tokens), _ptr(margin))
+    if st != ORACLE_OK:
+        raise OracleError(f"oracle_sample status {st}")
+    return probs, tokens, margin
+
+
+def lm_head_logits(hidden_bits, weight_bits):
+    """LM-head projection (Algorithm 1, the step before sampling): logits =
+    H W^T in float64 from bf16 hidden states H [R][hidden] and weights W
+    [V][hidden] (bf16 bit patterns, uint16), decoded exactly.  A library
+    matrix product is the only step."""
+    h = _bf16_to_f64(np.asarray(hidden_bits, np.uint16))
+    w = _bf16_to_f64(np.asarray(weight_bits, np.uint16))
+    return h @ w.T
+
+
+def _bf16_to_f64(bits):
+    return (np.asarray(bits, np.uint32) << 16).view(np.float32).astype(np.float64)

@@ -493,3 +493,71 @@ int oracle_kv_commit(int32_t *seq_lens, int32_t *block_table, int32_t *free_page
     *free_count = (int32_t)(top - taken);
     return ORACLE_OK;
 }
+
+/*
+ * 5. Draft tail sampling (Algorithm 1, last two steps: the LM head turns the
+ *    semi-autoregressive head's K hidden states into distributions
+ *    P'_1..P'_K, and T'_i ~ Categorical(P'_i); Sec. 3.3).  Given the fp32
+ *    logits of R rows: P' = softmax(logits / tau) (tau = the row's draft
+ *    temperature), and the token is drawn by inverse CDF with the row's
+ *    uniform u: the smallest x (ascending token id) with u * S < C(x),
+ *    C(x) = sum_{y <= x} exp((l_y - m) / tau), S = C(V - 1) (the same
+ *    convention as the residual draw of the acceptance); if rounding leaves
+ *    none, the last x with non-zero weight.  tau <= 0 is greedy drafting:
+ *    the token is the first argmax of the raw logits and P' is one-hot on it
+ *    (the limit of the softmax as tau -> 0 for a unique maximum).
+ *    margin[r] = min_x |u - C(x) / S| (0 for greedy rows): the distance of
+ *    the draw to the nearest CDF boundary.
+ */
+int oracle_sample(const float *logits, const float *uniforms, const float *temperature, int R,
+                  int V, double *probs, int32_t *tokens, double *margin)
+{
+    if (R < 1 || V < 1)
+        return ORACLE_ERR_ARG;
+    for (int r = 0; r < R; ++r) {
+        const float *row = logits + (size_t)r * V;
+        double *pr = probs + (size_t)r * V;
+        const double tau = temperature[r];
+        int best = 0;
+        for (int x = 1; x < V; ++x)
+            if (row[x] > row[best])
+                best = x;
+        if (!(tau > 0.0)) {
+            for (int x = 0; x < V; ++x)
+                pr[x] = 0.0;
+            pr[best] = 1.0;
+            tokens[r] = best;
+            if (margin)
+                margin[r] = 0.0;
+            continue;
+        }
+        const double m = (double)row[best] / tau;
+        double S = 0.0;
+        for (int x = 0; x < V; ++x) {
+            pr[x] = exp((double)row[x] / tau - m);
+            S += pr[x];
+        }
+        const double u = uniforms[r];
+        const double target = u * S;
+        double cdf = 0.0, nearest = INFINITY;
+        int tok = -1, last_positive = -1;
+        for (int x = 0; x < V; ++x) {
+            cdf += pr[x];
+            if (pr[x] > 0.0)
+                last_positive = x;
+            const double dist = fabs(u - cdf / S);
+            if (dist < nearest)
+                nearest = dist;
+            if (tok < 0 && target < cdf)
+                tok = x;
+        }
+        if (tok < 0)
+            tok = last_positive;
+        for (int x = 0; x < V; ++x)
+            pr[x] /= S;
+        tokens[r] = tok;
+        if (margin)
+            margin[r] = nearest;
+    }
+    return ORACLE_OK;
+}

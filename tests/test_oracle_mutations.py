@@ -51,6 +51,13 @@ MUTANTS = {
                                  "        for (long long lp = need; lp < had; ++lp) {\n            free_pages[sp++] = row[had - 1 - (lp - need)];"),
     "commit_page_count_floor": ("*need = (*next_len + page_size - 1) / page_size;",
                                 "*need = *next_len / page_size;"),
+    "sample_boundary_inclusive": ("            if (tok < 0 && target < cdf)\n                tok = x;",
+                                  "            if (tok < 0 && target <= cdf)\n                tok = x;"),
+    "sample_temperature_ignored": ("            pr[x] = exp((double)row[x] / tau - m);",
+                                   "            pr[x] = exp((double)row[x] - m * tau);"),
+    "sample_greedy_last_max": ("        for (int x = 1; x < V; ++x)\n            if (row[x] > row[best])\n                best = x;",
+                               "        for (int x = 1; x < V; ++x)\n            if (row[x] >= row[best])\n                best = x;"),
+    "sample_unnormalised_probs": ("            pr[x] /= S;", "            pr[x] /= 1.0;"),
 }
 
 
@@ -78,6 +85,7 @@ def test_pins_reject_mutant(name, source, tmp_path):
         [sys.executable, "-m", "pytest", "-x", "-q", "-p", "no:cacheprovider",
          os.path.join(ROOT, "tests", "test_oracle_attention.py"),
          os.path.join(ROOT, "tests", "test_oracle_accept.py"),
-         os.path.join(ROOT, "tests", "test_oracle_kv_commit.py")],
+         os.path.join(ROOT, "tests", "test_oracle_kv_commit.py"),
+         os.path.join(ROOT, "tests", "test_oracle_sample.py")],
         cwd=ROOT, env=env, capture_output=True, text=True, timeout=600)
     assert proc.returncode != 0, f"mutant {name} survived the oracle pins:\n{proc.stdout[-2000:]}"
