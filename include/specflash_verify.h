@@ -75,6 +75,8 @@ typedef enum {
 #define SF_MAX_QUERY_ROWS 16 /* n_q: draft rows scored per sequence           */
 #define SF_MAX_GROUP 8       /* H_q / H_kv                                    */
 #define SF_MAX_DRAFT 16      /* k: draft length                               */
+#define SF_MAX_DRAFT_ROWS 256 /* R: rows of one LM-head projection            */
+#define SF_MAX_VOCAB 8388608  /* V for sf_lm_head / sf_sample / sf_draft_sample */
 
 /* Static string naming a status code. */
 const char *sf_status_string(int status);
@@ -245,6 +247,57 @@ int sf_kv_commit(int32_t *seq_lens, int32_t *block_table, int32_t *free_pages,
                  int32_t *free_count, const int32_t *num_accepted, int B, int n_q, int n_q_next,
                  int max_pages_per_seq, int page_size, int capacity, void *workspace,
                  size_t workspace_bytes, cudaStream_t stream);
+
+/* ------------------------------------------------------------------------ */
+/* Draft-distribution tail (Sec. 3.3, Algorithm 1: the semi-autoregressive   */
+/* head's outputs for the K draft positions pass through the frozen LM head; */
+/* the K candidates are then sampled from the resulting distributions       */
+/* independently).  These calls produce the draft_probs / draft_tokens that  */
+/* sf_accept consumes (rows R = B * k, row b * k + i for draft position i). */
+/*                                                                           */
+/* sf_lm_head:  logits[r][v] = sum_j hidden[r][j] * weight[v][j], bf16       */
+/*              inputs, fp32 accumulation (tensor cores), fp32 output.       */
+/* sf_sample:   for each row r, with tau = temperature[r]:                   */
+/*              probs[r] = softmax(logits[r] / tau), and tokens[r] = the     */
+/*              smallest token x with uniforms[r] * S < C(x), where C is the */
+/*              cumulative sum of exp(logits/tau - max) in ascending token   */
+/*              order and S its total; tau <= 0 (or NaN) selects greedy      */
+/*              decoding: tokens[r] = the first argmax, probs[r] one-hot.    */
+/*              Tokens at -inf get probability 0.  Where rounding leaves no  */
+/*              token past the target (uniforms[r] >= 1 or NaN), the last    */
+/*              token of positive probability is taken.                      */
+/* sf_draft_sample: sf_lm_head then sf_sample, with the per-row max and sum  */
+/*              reduced in the projection's epilogue, so the logits are read */
+/*              once more (for probs) instead of three times.                */
+/*                                                                           */
+/* hidden       bf16 [R][hidden_size], 16-byte aligned.                      */
+/* weight       bf16 [V][hidden_size] (the LM head), 16-byte aligned.        */
+/*              hidden_size a multiple of 8 in [8, 2^20]; 1 <= R <= 256      */
+/*              (sf_sample alone: R <= 65535); 1 <= V <= SF_MAX_VOCAB.       */
+/* logits       fp32 [R][V]: output of sf_lm_head / sf_draft_sample, input   */
+/*              of sf_sample.                                                */
+/* uniforms     fp32 [R] in [0, 1).   temperature  fp32 [R].                 */
+/* probs        fp32 [R][V].          tokens       int32 [R].                */
+/* workspace    >= sf_draft_tail_workspace_size(R, V) bytes, 256-byte        */
+/*              aligned, zero-filled before first use (status word).        */
+/* Stream order: the projection copies weight tiles before waiting for the   */
+/* previous kernel on the stream (the weights must not be written by it);    */
+/* hidden, temperature, uniforms and the outputs follow it.                  */
+/* Results are deterministic; SF_DEVICE_TIMEOUT is the only device status.   */
+/* ------------------------------------------------------------------------ */
+size_t sf_draft_tail_workspace_size(int R, int V);
+
+int sf_lm_head(const void *hidden, const void *weight, int R, int hidden_size, int V,
+               float *logits, void *workspace, size_t workspace_bytes, cudaStream_t stream);
+
+int sf_sample(const float *logits, const float *uniforms, const float *temperature, int R, int V,
+              float *probs, int32_t *tokens, void *workspace, size_t workspace_bytes,
+              cudaStream_t stream);
+
+int sf_draft_sample(const void *hidden, const void *weight, const float *uniforms,
+                    const float *temperature, int R, int hidden_size, int V, float *logits,
+                    float *probs, int32_t *tokens, void *workspace, size_t workspace_bytes,
+                    cudaStream_t stream);
 
 #ifdef __cplusplus
 }

@@ -31,6 +31,7 @@ EXPORTED_SYMBOLS = (
     "sf_verify_attention_noalloc",
     "sf_accept_workspace_size", "sf_accept",
     "sf_kv_commit_workspace_size", "sf_kv_commit",
+    "sf_draft_tail_workspace_size", "sf_lm_head", "sf_sample", "sf_draft_sample",
 )
 
 _lock = threading.Lock()
@@ -87,6 +88,14 @@ def load_library(path: str | None = None):
         lib.sf_kv_commit_workspace_size.restype = S
         lib.sf_kv_commit.argtypes = [P, P, P, P, P, I, I, I, I, I, I, P, S, P]
         lib.sf_kv_commit.restype = I
+        lib.sf_draft_tail_workspace_size.argtypes = [I, I]
+        lib.sf_draft_tail_workspace_size.restype = S
+        lib.sf_lm_head.argtypes = [P, P, I, I, I, P, P, S, P]
+        lib.sf_lm_head.restype = I
+        lib.sf_sample.argtypes = [P, P, P, I, I, P, P, P, S, P]
+        lib.sf_sample.restype = I
+        lib.sf_draft_sample.argtypes = [P, P, P, P, I, I, I, P, P, P, P, S, P]
+        lib.sf_draft_sample.restype = I
         _lib = lib
         return lib
 
@@ -281,3 +290,82 @@ def kv_commit(seq_lens, block_table, free_pages, free_count, num_accepted, n_q, 
         _ptr(seq_lens), _ptr(block_table), _ptr(free_pages), _ptr(free_count), _ptr(num_accepted),
         B, n_q, n_q_next, max_pages, PAGE_SIZE, free_pages.numel(), _ptr(workspace),
         workspace.numel(), _stream_handle(stream)))
+
+
+# --------------------------------------------------------------------------- #
+# draft-distribution tail                                                     #
+# --------------------------------------------------------------------------- #
+def draft_tail_workspace_size(R, V) -> int:
+    n = load_library().sf_draft_tail_workspace_size(R, V)
+    if n == 0:
+        raise SFError(1, "invalid draft-tail shape: " + load_library().sf_last_error().decode())
+    return int(n)
+
+
+def lm_head(hidden, weight, *, logits=None, workspace=None, stream=None):
+    """sf_lm_head: hidden bf16 [R][hidden_size], weight bf16 [V][hidden_size].
+    Returns logits fp32 [R][V] = hidden @ weight^T."""
+    R, Hd = hidden.shape
+    V = weight.shape[0]
+    _need(hidden, "hidden", torch.bfloat16)
+    _need(weight, "weight", torch.bfloat16, (V, Hd))
+    if logits is None:
+        logits = torch.empty((R, V), dtype=torch.float32, device=hidden.device)
+    _need(logits, "logits", torch.float32, (R, V))
+    if workspace is None:
+        workspace = new_workspace(draft_tail_workspace_size(R, V), hidden.device)
+    _check(load_library().sf_lm_head(_ptr(hidden), _ptr(weight), R, Hd, V, _ptr(logits),
+                                     _ptr(workspace), workspace.numel(), _stream_handle(stream)))
+    return logits
+
+
+def sample(logits, uniforms, temperature, *, probs=None, tokens=None, workspace=None,
+           stream=None):
+    """sf_sample: logits fp32 [R][V], uniforms fp32 [R], temperature fp32 [R]
+    (<= 0 greedy).  Returns (probs fp32 [R][V], tokens int32 [R])."""
+    R, V = logits.shape
+    _need(logits, "logits", torch.float32)
+    _need(uniforms, "uniforms", torch.float32, (R,))
+    _need(temperature, "temperature", torch.float32, (R,))
+    dev = logits.device
+    if probs is None:
+        probs = torch.empty((R, V), dtype=torch.float32, device=dev)
+    if tokens is None:
+        tokens = torch.empty(R, dtype=torch.int32, device=dev)
+    _need(probs, "probs", torch.float32, (R, V))
+    _need(tokens, "tokens", torch.int32, (R,))
+    if workspace is None:
+        workspace = new_workspace(draft_tail_workspace_size(R, V), dev)
+    _check(load_library().sf_sample(_ptr(logits), _ptr(uniforms), _ptr(temperature), R, V,
+                                    _ptr(probs), _ptr(tokens), _ptr(workspace), workspace.numel(),
+                                    _stream_handle(stream)))
+    return probs, tokens
+
+
+def draft_sample(hidden, weight, uniforms, temperature, *, logits=None, probs=None, tokens=None,
+                 workspace=None, stream=None):
+    """sf_draft_sample: the LM-head projection and sampling of the draft
+    rows in two launches.  Returns (logits fp32 [R][V], probs fp32 [R][V],
+    tokens int32 [R])."""
+    R, Hd = hidden.shape
+    V = weight.shape[0]
+    _need(hidden, "hidden", torch.bfloat16)
+    _need(weight, "weight", torch.bfloat16, (V, Hd))
+    _need(uniforms, "uniforms", torch.float32, (R,))
+    _need(temperature, "temperature", torch.float32, (R,))
+    dev = hidden.device
+    if logits is None:
+        logits = torch.empty((R, V), dtype=torch.float32, device=dev)
+    if probs is None:
+        probs = torch.empty((R, V), dtype=torch.float32, device=dev)
+    if tokens is None:
+        tokens = torch.empty(R, dtype=torch.int32, device=dev)
+    _need(logits, "logits", torch.float32, (R, V))
+    _need(probs, "probs", torch.float32, (R, V))
+    _need(tokens, "tokens", torch.int32, (R,))
+    if workspace is None:
+        workspace = new_workspace(draft_tail_workspace_size(R, V), dev)
+    _check(load_library().sf_draft_sample(
+        _ptr(hidden), _ptr(weight), _ptr(uniforms), _ptr(temperature), R, Hd, V, _ptr(logits),
+        _ptr(probs), _ptr(tokens), _ptr(workspace), workspace.numel(), _stream_handle(stream)))
+    return logits, probs, tokens

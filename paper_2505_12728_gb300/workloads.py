@@ -248,3 +248,89 @@ def make_accept_inputs(wl: Workload, seed=None, mode=None) -> AcceptInputs:
     seed = wl.seed if seed is None else seed
     return make_accept_case(wl.B, wl.k, wl.V, seed=[seed, 0xACC], mode=mode or wl.mode,
                             draft_sharpness=wl.draft_sharpness, logit_std=wl.logit_std)
+
+
+# --------------------------------------------------------------------------- #
+# draft-tail inputs                                                           #
+# --------------------------------------------------------------------------- #
+# Hidden sizes of the target/draft LM heads: LLaVA-1.5-7B (Vicuna-7B) for the
+# 32000-token vocabulary, Qwen2-VL-7B for the 152064-token one.
+HIDDEN_SIZES = {32000: 4096, 152064: 3584}
+
+
+@dataclass
+class DraftTailInputs:
+    hidden: np.ndarray       # uint16 bf16 bits [R][hidden_size]: draft head outputs
+    weight: np.ndarray       # uint16 bf16 bits [V][hidden_size]: the LM head
+    uniforms: np.ndarray     # fp32 [R]
+    temperature: np.ndarray  # fp32 [R]
+
+    @property
+    def shape(self):
+        return self.hidden.shape[0], self.hidden.shape[1], self.weight.shape[0]
+
+
+def _scaled_normal_bf16(rng: np.random.Generator, shape, std: float) -> np.ndarray:
+    n = int(np.prod(shape))
+    out = np.empty(n, np.uint16)
+    chunk = 1 << 24
+    for s in range(0, n, chunk):
+        e = min(n, s + chunk)
+        out[s:e] = f32_to_bf16_bits(np.float32(std) * rng.standard_normal(e - s, dtype=np.float32))
+    return out.reshape(shape)
+
+
+def _small_int_bf16(rng: np.random.Generator, shape, scale: float) -> np.ndarray:
+    n = int(np.prod(shape))
+    out = np.empty(n, np.uint16)
+    chunk = 1 << 24
+    for s in range(0, n, chunk):
+        e = min(n, s + chunk)
+        v = rng.integers(-3, 4, size=e - s).astype(np.float32) * np.float32(scale)
+        out[s:e] = f32_to_bf16_bits(v)
+    return out.reshape(shape)
+
+
+def make_draft_tail_case(R, hidden_size, V, seed, temperature=None, logit_std=3.0, exact=False):
+    """Hidden states ~ N(0,1) and LM-head weights ~ N(0, logit_std^2 /
+    hidden_size), both rounded to bf16, so the logits are ~ N(0, logit_std^2)
+    like the target logits of the acceptance inputs; uniforms ~ U[0,1);
+    temperature per row (default 1).
+
+    exact=True draws both from the integers -3..3 instead, the weights scaled
+    by a power of two 2^-e (logit std within a factor 2 of logit_std): every
+    product and partial sum is then a multiple of 2^-e below 2^24 * 2^-e, so
+    any fp32 accumulation order gives the exact logits."""
+    rng = np.random.default_rng(seed)
+    if exact:
+        e = int(np.floor(np.log2(4.0 * np.sqrt(hidden_size) / logit_std)))
+        hidden = _small_int_bf16(rng, (R, hidden_size), 1.0)
+        weight = _small_int_bf16(rng, (V, hidden_size), 2.0 ** -e)
+    else:
+        hidden = _normal_bf16(rng, (R, hidden_size))
+        weight = _scaled_normal_bf16(rng, (V, hidden_size), logit_std / np.sqrt(hidden_size))
+    uniforms = rng.random(R, dtype=np.float32)
+    if temperature is None:
+        temperature = np.ones(R, np.float32)
+    temperature = np.asarray(temperature, np.float32).reshape(R)
+    return DraftTailInputs(hidden=hidden, weight=weight, uniforms=uniforms, temperature=temperature)
+
+
+def make_draft_tail_inputs(wl: Workload, seed=None, exact=False) -> DraftTailInputs:
+    """The K = wl.k draft positions of each of the B sequences (row b*k + i),
+    each sequence at its workload temperature."""
+    seed = wl.seed if seed is None else seed
+    temp = np.repeat(temperatures(wl.mode, wl.B), wl.k)
+    return make_draft_tail_case(wl.B * wl.k, HIDDEN_SIZES[wl.V], wl.V, seed=[seed, 0xD4AF7],
+                                temperature=temp, logit_std=wl.logit_std, exact=exact)
+
+
+def make_sample_case(R, V, seed, temperature=None, logit_std=3.0):
+    """fp32 logits ~ N(0, logit_std^2) [R][V] and uniforms ~ U[0,1) [R] for
+    the sampler alone."""
+    rng = np.random.default_rng(seed)
+    logits = (logit_std * rng.standard_normal((R, V), dtype=np.float32)).astype(np.float32)
+    uniforms = rng.random(R, dtype=np.float32)
+    if temperature is None:
+        temperature = np.ones(R, np.float32)
+    return logits, uniforms, np.asarray(temperature, np.float32).reshape(R)
