@@ -154,9 +154,14 @@ KERNEL_SOURCES = {
     "verify_attention_tc_kernel": ["paper_2505_12728_gb300/csrc/verify_attention_tc.cu",
                                    "paper_2505_12728_gb300/csrc/attn_common.cuh",
                                    "paper_2505_12728_gb300/csrc/sf_device.cuh"],
+    "lm_head_kernel": ["paper_2505_12728_gb300/csrc/draft_tail.cu",
+                       "paper_2505_12728_gb300/csrc/ff_math.cuh",
+                       "paper_2505_12728_gb300/csrc/sf_device.cuh"],
 }
 PROFILES = {"image7b": "profiles/verify_attention_image7b.md",
             "video": "profiles/verify_attention_tc_video.md"}
+LM_HEAD_PROFILES = {"image7b": "profiles/lm_head_image7b.md",
+                    "long": "profiles/lm_head_long.md"}
 
 
 def attention_kernel(wl):
@@ -279,6 +284,64 @@ def run_reference(args):
                     "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
     return 0
+
+
+def time_draft_tail(wl, dev, stream, capture):
+    """Device time of sf_draft_sample (projection + sampling) and of
+    sf_lm_head alone for the workload's B*k draft rows over a random bf16 LM
+    head of the target's shape (V x hidden), each replayed from a CUDA graph
+    of 10 calls; the weights (262 MB-1.09 GB) exceed L2, so every call
+    streams them from HBM."""
+    import torch
+    from paper_2505_12728_gb300 import specflash_verify as sfv
+    from paper_2505_12728_gb300.workloads import make_draft_tail_inputs
+    case = make_draft_tail_inputs(wl)
+    R, Hd, V = case.shape
+    bf = lambda bits: torch.from_numpy(np.ascontiguousarray(bits).view(np.int16)).to(dev).view(
+        torch.bfloat16)
+    h, w = bf(case.hidden), bf(case.weight)
+    u = torch.from_numpy(case.uniforms).to(dev)
+    t = torch.from_numpy(case.temperature).to(dev)
+    logits = torch.empty((R, V), dtype=torch.float32, device=dev)
+    probs = torch.empty_like(logits)
+    tokens = torch.empty(R, dtype=torch.int32, device=dev)
+    ws = sfv.new_workspace(sfv.draft_tail_workspace_size(R, V), dev)
+    fused = lambda: sfv.draft_sample(h, w, u, t, logits=logits, probs=probs, tokens=tokens,
+                                     workspace=ws, stream=stream)
+    proj = lambda: sfv.lm_head(h, w, logits=logits, workspace=ws, stream=stream)
+
+    def per_call_us(fn, calls=10, reps=5):
+        fn()
+        g = capture(lambda: [fn() for _ in range(calls)])
+        g.replay()
+        a = torch.cuda.Event(enable_timing=True)
+        b = torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        for _ in range(reps):
+            g.replay()
+        b.record(stream)
+        torch.cuda.synchronize()
+        return a.elapsed_time(b) * 1e3 / (calls * reps)
+
+    fused_us = per_call_us(fused)
+    proj_us = per_call_us(proj)
+    status = sfv.read_device_status(ws)
+    ok = bool(torch.isfinite(probs).all().item()) and \
+        float((probs.double().sum(1) - 1).abs().max().item()) < 1e-5
+    peak, kind = measured_peaks()
+    alg = V * Hd * 2 + R * Hd * 2 + R * V * 4  # weights + hidden states + logits
+    gbs = alg / (proj_us * 1e-6) / 1e9
+    del w
+    return {"rows": R, "hidden": Hd, "vocab": V, "draft_sample_us": fused_us,
+            "lm_head_us": proj_us, "sampling_us": fused_us - proj_us,
+            "lm_head_gbs": gbs, "lm_head_frac": gbs / peak,
+            "lm_head_algorithmic_bytes": alg,
+            "lm_head_traffic": (profiled_traffic(KERNEL_SOURCES["lm_head_kernel"],
+                                                 LM_HEAD_PROFILES[wl.name])
+                                if wl.name in LM_HEAD_PROFILES else None),
+            "peak_gbs": peak, "peak_source": kind,
+            "kernels": ["lm_head_kernel", "sample_finish_kernel"],
+            "probs_sum_to_one": ok, "device_status": status}
 
 
 def workload_config(wl, seq_lens):
@@ -444,6 +507,10 @@ def run_ours(args):
         commit_us = c0.elapsed_time(c1) * 1e3 / 500
         assert sfv.read_device_status(c_ws) == 0 and torch.equal(c_sl, sl)
 
+    # ---- draft-distribution tail (the LM head, softmax and sampling of the
+    # B*k draft rows that produce q and T'; outside the verification step)
+    dt = time_draft_tail(wl, dev, stream, capture) if not args.no_draft_tail else None
+
     # ---- end to end through host buffers ----
     pin = lambda a: torch.from_numpy(np.ascontiguousarray(a)).pin_memory()
     h_q = pin(att.q.view(np.int16))
@@ -509,6 +576,7 @@ def run_ours(args):
         "kv_frac_of_nominal_8tbs": achieved / NOMINAL_HBM_GBS,
         "accept_gbs": accept_bytes(wl, sampling_rows) / (acc_launch_ms / 1e3) / 1e9,
         "kv_commit_us": commit_us,
+        "draft_tail": dt,
         "mean_accepted": float(n_acc.float().mean().item()),
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                      "frac": achieved / peak,
@@ -549,6 +617,8 @@ def main(argv=None):
     ap.add_argument("--cpu-budget", type=float, default=12.0,
                     help="seconds of oracle work for the cpu_baseline sample")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-draft-tail", action="store_true",
+                    help="skip the draft-tail (LM head + sampling) timing")
     ap.add_argument("--eager", action="store_true",
                     help="launch every call from Python instead of replaying CUDA graphs")
     args = ap.parse_args(argv)
