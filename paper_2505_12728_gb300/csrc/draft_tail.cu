@@ -12,8 +12,11 @@
 // (262 MB for LLaVA's 32000 x 4096, 1.09 GB for QwenVL's 152064 x 3584) for
 // a few dozen rows, so it is bound by HBM and everything else hides under
 // that stream:
-//  * lm_head_kernel: one CTA per SM, each owning a contiguous range of
-//    128-token vocabulary tiles.  Warp 5 streams 128 x 64 weight boxes and
+//  * lm_head_kernel: one CTA per SM, each owning an equal contiguous range
+//    of vocabulary rows (floor or ceil of V / G), cut into 128-row tiles; a
+//    range's last tile is loaded with a box of exactly its remaining height
+//    (two extra tensor maps), so every SM streams the same number of weight
+//    bytes.  Warp 5 streams 128 x 64 weight boxes and
 //    the matching 64-column box of the hidden states (rows padded to NP, a
 //    multiple of 16, by the copy's zero fill) into a deep ring; warp 4 issues
 //    logits^T = W H^T as tcgen05 MMAs of M = 128 (vocabulary), N = NP (draft
@@ -63,7 +66,7 @@ constexpr int kLmColGroup = 16;                        // draft rows per epilogu
 constexpr int kLmTStride = 136;                        // floats per transposed row (8 mod 32 banks)
 constexpr int kLmTBufFloats = 2 * kLmColGroup * kLmTStride;
 constexpr int kSampleUnit = 2048;                      // tokens per statistics chunk (sf_sample)
-constexpr int kSampleSpan = 4096;                      // tokens per finishing CTA
+constexpr int kSampleSpan = 4096;                      // least tokens per finishing CTA
 constexpr int kMaxStatChunks = 4096;                   // statistics chunks per row
 
 struct SampStat {  // one chunk of one row
@@ -79,8 +82,8 @@ struct LmParams {
   SampStat *stats;   // [R][G], or null for the plain projection
   uint32_t *status;
   int R, V, NP;
-  int T;             // vocabulary tiles
-  int G;             // CTAs; CTA c owns tiles [c*T/G, (c+1)*T/G)
+  int G;             // CTAs; CTA c owns vocabulary rows [c*V/G, (c+1)*V/G)
+  int ha, hb;        // box heights of the two last-tile weight maps
   int KC;            // hidden chunks of 64
   int stages;
   uint32_t stage_bytes;  // weight box + NP * 128 bytes of hidden states
@@ -98,6 +101,7 @@ struct SampleParams {
   int R, V;
   int Cn;                 // statistics chunks per row
   int unit, T;            // chunk c covers [e(c), e(c+1)), e(c) = min(V, unit * (c*T/Cn))
+  int span;               // tokens per finishing CTA (a multiple of 4)
   int vec4;               // rows 16-byte aligned and V % 4 == 0
 };
 
@@ -132,7 +136,8 @@ __device__ __forceinline__ void stat_merge(SampStat &run, float m, int arg, ff s
 }
 
 __global__ void __launch_bounds__(kLmThreads, 1)
-lm_head_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant__ CUtensorMap tmap_h,
+lm_head_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant__ CUtensorMap tmap_wa,
+               const __grid_constant__ CUtensorMap tmap_wb, const __grid_constant__ CUtensorMap tmap_h,
                const __grid_constant__ LmParams p) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t *smem = reinterpret_cast<uint8_t *>(
@@ -151,10 +156,17 @@ lm_head_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
   auto bar = [&](int i) -> uint32_t { return bars + 8u * static_cast<uint32_t>(i); };
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int t0 = static_cast<int>(static_cast<long long>(blockIdx.x) * p.T / p.G);
-  const int t1 = static_cast<int>(static_cast<long long>(blockIdx.x + 1) * p.T / p.G);
-  const int n_tiles = t1 - t0;
+  const int v0 = static_cast<int>(static_cast<long long>(blockIdx.x) * p.V / p.G);
+  const int v1 = static_cast<int>(static_cast<long long>(blockIdx.x + 1) * p.V / p.G);
+  const int n_tiles = (v1 - v0 + kLmTileV - 1) / kLmTileV;
+  const int last_h = v1 - v0 - (n_tiles - 1) * kLmTileV;  // rows of the last tile
   const uint32_t total = static_cast<uint32_t>(n_tiles) * static_cast<uint32_t>(p.KC);
+  // weight map and box height of tile i
+  auto tile_map = [&](int i, uint32_t &bytes) -> const CUtensorMap * {
+    const int h = i == n_tiles - 1 ? last_h : kLmTileV;
+    bytes = static_cast<uint32_t>(h) * (kLmChunkK * 2) + static_cast<uint32_t>(p.NP) * (kLmChunkK * 2);
+    return h == kLmTileV ? &tmap_w : (h == p.ha ? &tmap_wa : &tmap_wb);
+  };
 
   grid_launch_dependents();
   if (tid == 0) {
@@ -169,6 +181,8 @@ lm_head_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
     mbar_init(bar(FIN), 1);
     fence_mbar_init();
     prefetch_tensormap(&tmap_w);
+    prefetch_tensormap(&tmap_wa);
+    prefetch_tensormap(&tmap_wb);
     prefetch_tensormap(&tmap_h);
     s_misc[1] = 0;
     s_misc[2] = 0;
@@ -192,9 +206,11 @@ lm_head_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
       // states (possibly written by the previous kernel) after it
       for (uint32_t q = 0; q < prime; ++q) {
         const int i = static_cast<int>(q) / p.KC, kc = static_cast<int>(q) % p.KC;
-        mbar_arrive_expect_tx(bar(FULL + q), p.stage_bytes);
-        tma_load_2d(ring + q * p.stage_bytes, &tmap_w, kc * kLmChunkK, (t0 + i) * kLmTileV,
-                    bar(FULL + q), pol_w);
+        uint32_t bytes;
+        const CUtensorMap *mw = tile_map(i, bytes);
+        mbar_arrive_expect_tx(bar(FULL + q), bytes);
+        tma_load_2d(ring + q * p.stage_bytes, mw, kc * kLmChunkK, v0 + i * kLmTileV, bar(FULL + q),
+                    pol_w);
       }
       grid_dependency_wait();
       for (uint32_t q = 0; q < prime; ++q) {
@@ -208,8 +224,10 @@ lm_head_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
         if (!mbar_wait_or_abort(bar(EMPTY + slot), ((q / S) - 1) & 1u, s_abort)) break;
         const int i = static_cast<int>(q / p.KC), kc = static_cast<int>(q % p.KC);
         const uint32_t dst = ring + slot * p.stage_bytes;
-        mbar_arrive_expect_tx(bar(FULL + slot), p.stage_bytes);
-        tma_load_2d(dst, &tmap_w, kc * kLmChunkK, (t0 + i) * kLmTileV, bar(FULL + slot), pol_w);
+        uint32_t bytes;
+        const CUtensorMap *mw = tile_map(i, bytes);
+        mbar_arrive_expect_tx(bar(FULL + slot), bytes);
+        tma_load_2d(dst, mw, kc * kLmChunkK, v0 + i * kLmTileV, bar(FULL + slot), pol_w);
         tma_load_2d(dst + kLmWBytes, &tmap_h, kc * kLmChunkK, 0, bar(FULL + slot), pol_h);
       }
       s_misc[2] = static_cast<int>(q);
@@ -219,6 +237,8 @@ lm_head_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
     // ------------------------------------------------------------------
     // MMA issue: per 64-column chunk four MMAs (K = 16 each, +32 bytes
     // along the 128-byte swizzled rows); the slot is released by a commit.
+    // Rows of a short last tile beyond its box hold stale data; their
+    // accumulator rows are never stored.
     // ------------------------------------------------------------------
     uint32_t q = 0;
     bool ok = true;
@@ -285,9 +305,9 @@ lm_head_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
       bool ok = mbar_wait_or_abort(bar(DFULL + buf), (i >> 1) & 1, s_abort);
       if (!named_bar_and(2, kLmEpiThreads, ok)) break;
       tc_fence_after_sync();
-      const int vbase = (t0 + i) * kLmTileV;
+      const int vbase = v0 + i * kLmTileV;
       const int v = vbase + 32 * warp + lane;
-      const bool vin = v < p.V;
+      const bool vin = v < v1;
       for (int g = 0; g < groups; ++g, ++g_count) {
         const int c0 = g * kLmColGroup;
         uint32_t x[16];
@@ -421,8 +441,8 @@ __global__ void __launch_bounds__(kFfThreads) sample_stats_kernel(const __grid_c
 }
 
 // Combines a row's chunk statistics, writes P' for this CTA's span of
-// kSampleSpan tokens and, in the CTA holding the crossing chunk's first
-// token, draws T'.  grid (ceil(V / kSampleSpan), R); dynamic shared memory
+// tokens and, in the CTA holding the crossing chunk's first
+// token, draws T'.  grid (ceil(V / span), R); dynamic shared memory
 // holds the row's Cn statistics.
 __global__ void __launch_bounds__(kFfThreads) sample_finish_kernel(const __grid_constant__ SampleParams p) {
   extern __shared__ SampStat s_st[];
@@ -456,8 +476,8 @@ __global__ void __launch_bounds__(kFfThreads) sample_finish_kernel(const __grid_
   block_argmax(m, arg, s_v, s_i);
 
   const float tau = p.tau[r];
-  const int x0 = blockIdx.x * kSampleSpan;
-  const int x1 = min(p.V, x0 + kSampleSpan);
+  const int x0 = blockIdx.x * p.span;
+  const int x1 = min(p.V, x0 + p.span);
   if (!(tau > 0.f)) {
     // greedy: one-hot P', T' = the first argmax
     for (int x = x0 + tid; x < x1; x += kFfThreads) prow[x] = x == arg ? 1.f : 0.f;
@@ -501,20 +521,31 @@ __global__ void __launch_bounds__(kFfThreads) sample_finish_kernel(const __grid_
   const bool crossed = s_c != INT_MAX;
   const int cs = crossed ? s_c : s_last;  // no crossing (u >= 1 or NaN): last positive chunk
 
-  // P' for this CTA's span
+  // P' for this CTA's span.  Rows are 16-byte aligned and the span a
+  // multiple of 4 in the vector path, so a float4 is either wholly inside
+  // the span or wholly outside; each thread issues kBatch loads before
+  // the arithmetic and stores that depend on them.
   const float invS = ff_div_to_f(1.f, Stot);
   if (p.vec4) {
-    for (int x = x0 + 4 * tid; x < x1; x += 4 * kFfThreads) {
-      if (x + 3 < x1) {
-        const float4 f = *reinterpret_cast<const float4 *>(row + x);
-        float4 o;
-        o.x = __fmul_rn(term_of(f.x, m, tau), invS);
-        o.y = __fmul_rn(term_of(f.y, m, tau), invS);
-        o.z = __fmul_rn(term_of(f.z, m, tau), invS);
-        o.w = __fmul_rn(term_of(f.w, m, tau), invS);
-        *reinterpret_cast<float4 *>(prow + x) = o;
-      } else {
-        for (int j = x; j < x1; ++j) prow[j] = __fmul_rn(term_of(row[j], m, tau), invS);
+    constexpr int kBatch = 4;
+    for (int base = x0 + 4 * tid; base < x1; base += 4 * kFfThreads * kBatch) {
+      float4 f[kBatch];
+#pragma unroll
+      for (int j = 0; j < kBatch; ++j) {
+        const int x = base + j * 4 * kFfThreads;
+        if (x < x1) f[j] = __ldcs(reinterpret_cast<const float4 *>(row + x));
+      }
+#pragma unroll
+      for (int j = 0; j < kBatch; ++j) {
+        const int x = base + j * 4 * kFfThreads;
+        if (x < x1) {
+          float4 o;
+          o.x = __fmul_rn(term_of(f[j].x, m, tau), invS);
+          o.y = __fmul_rn(term_of(f[j].y, m, tau), invS);
+          o.z = __fmul_rn(term_of(f[j].z, m, tau), invS);
+          o.w = __fmul_rn(term_of(f[j].w, m, tau), invS);
+          *reinterpret_cast<float4 *>(prow + x) = o;
+        }
       }
     }
   } else {
@@ -591,8 +622,9 @@ static int lm_setup(const DeviceInfo &dev) {
   return SF_OK;
 }
 
-// Tensor maps of the weights {hidden, V} (box 64 x 128) and hidden states
-// {hidden, R} (box 64 x NP), cached by (base, rows, hidden, box rows).
+// Tensor maps of the weights {hidden, V} (box 64 x 128, 64 x ha, 64 x hb) and
+// hidden states {hidden, R} (box 64 x NP), cached by (base, rows, hidden, box
+// rows).
 static int lm_tensor_map(CUtensorMap *out, const void *base, uint64_t rows, int hidden, uint32_t box_rows) {
   static std::mutex mu;
   static std::map<std::tuple<const void *, uint64_t, int, uint32_t>, CUtensorMap> maps;
@@ -681,8 +713,11 @@ static int launch_lm_head(const void *hidden, const void *weight, int R, int hid
   prm.R = R;
   prm.V = V;
   prm.NP = NP;
-  prm.T = (V + kLmTileV - 1) / kLmTileV;
-  prm.G = prm.T < dev.sm_count ? prm.T : dev.sm_count;
+  const int tiles = (V + kLmTileV - 1) / kLmTileV;
+  prm.G = tiles < dev.sm_count ? tiles : dev.sm_count;
+  const int q = V / prm.G;  // every CTA owns q or q + 1 rows
+  prm.ha = (q - 1) % kLmTileV + 1;
+  prm.hb = q % kLmTileV + 1;
   prm.KC = (hidden_size + kLmChunkK - 1) / kLmChunkK;
   prm.stage_bytes = kLmWBytes + static_cast<uint32_t>(NP) * 128u;
   prm.stages = lm_stages(dev, prm.stage_bytes, NP);
@@ -693,22 +728,39 @@ static int launch_lm_head(const void *hidden, const void *weight, int R, int hid
   const size_t smem = LmSmem::bytes(prm.stages, prm.stage_bytes, NP);
   if (smem > static_cast<size_t>(dev.max_smem_optin))
     return fail(SF_ERR_UNSUPPORTED, "LM-head ring needs %zu bytes of shared memory", smem);
-  CUtensorMap tw, th;
+  CUtensorMap tw, twa, twb, th;
   st = lm_tensor_map(&tw, weight, static_cast<uint64_t>(V), hidden_size, kLmTileV);
+  if (st == SF_OK)
+    st = lm_tensor_map(&twa, weight, static_cast<uint64_t>(V), hidden_size, static_cast<uint32_t>(prm.ha));
+  if (st == SF_OK)
+    st = lm_tensor_map(&twb, weight, static_cast<uint64_t>(V), hidden_size, static_cast<uint32_t>(prm.hb));
   if (st != SF_OK) return st;
   st = lm_tensor_map(&th, hidden, static_cast<uint64_t>(R), hidden_size, static_cast<uint32_t>(NP));
   if (st != SF_OK) return st;
   cudaLaunchAttribute attr[1];
   cudaLaunchConfig_t cfg = pdl_config(dim3(prm.G), dim3(kLmThreads), smem, stream, attr);
-  cudaError_t e = cudaLaunchKernelEx(&cfg, lm_head_kernel, tw, th, prm);
+  cudaError_t e = cudaLaunchKernelEx(&cfg, lm_head_kernel, tw, twa, twb, th, prm);
   if (e != cudaSuccess) return fail(SF_ERR_CUDA, "LM-head launch: %s", cudaGetErrorString(e));
   if (G_out) *G_out = prm.G;
   return SF_OK;
 }
 
-static int launch_finish(const SampleParams &prm, cudaStream_t stream) {
+// Span per finishing CTA: about one wave of CTAs (8 per SM) over all rows,
+// at least kSampleSpan tokens, a multiple of kSampleSpan.
+static int finish_span(int R, int V) {
+  DeviceInfo dev;
+  const int sms = current_device(&dev) == SF_OK ? dev.sm_count : 148;
+  const long long per = ((long long)R * V + 8LL * sms - 1) / (8LL * sms);
+  long long span = (per + kSampleSpan - 1) / kSampleSpan * kSampleSpan;
+  if (span < kSampleSpan) span = kSampleSpan;
+  if (span > V) span = (V + 3) / 4 * 4;
+  return static_cast<int>(span);
+}
+
+static int launch_finish(SampleParams prm, cudaStream_t stream) {
   cudaLaunchAttribute attr[1];
-  const int spans = (prm.V + kSampleSpan - 1) / kSampleSpan;
+  prm.span = finish_span(prm.R, prm.V);
+  const int spans = (prm.V + prm.span - 1) / prm.span;
   cudaLaunchConfig_t cfg = pdl_config(dim3(spans, prm.R), dim3(kFfThreads),
                                       static_cast<size_t>(prm.Cn) * sizeof(SampStat), stream, attr);
   cudaError_t e = cudaLaunchKernelEx(&cfg, sample_finish_kernel, prm);
@@ -809,9 +861,9 @@ int sf_draft_sample(const void *hidden, const void *weight, const float *uniform
   prm.tokens = tokens;
   prm.R = R;
   prm.V = V;
-  prm.Cn = G;
-  prm.unit = kLmTileV;
-  prm.T = (V + kLmTileV - 1) / kLmTileV;
+  prm.Cn = G;  // chunk c = CTA c's rows [c*V/G, (c+1)*V/G)
+  prm.unit = 1;
+  prm.T = V;
   prm.vec4 = (V % 4 == 0) && aligned(logits, 16) && aligned(probs, 16);
   return launch_finish(prm, stream);
 }
