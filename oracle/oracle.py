@@ -76,6 +76,8 @@ def _load():
         lib.oracle_kv_commit.restype = I
         lib.oracle_sample.argtypes = [P, P, P, I, I, P, P, P]
         lib.oracle_sample.restype = I
+        lib.oracle_visual_compress.argtypes = [P, P, I, I, I, I, P]
+        lib.oracle_visual_compress.restype = I
         _lib = lib
         return lib
 
@@ -251,6 +253,26 @@ def lm_head_logits(hidden_bits, weight_bits):
     h = _bf16_to_f64(np.asarray(hidden_bits, np.uint16))
     w = _bf16_to_f64(np.asarray(weight_bits, np.uint16))
     return h @ w.T
+
+
+def visual_compress(query_bits, feature_bits):
+    """Visual token compression (Sec. 3.2, Eq. 3; Algorithm 1):
+    F^_V = softmax(Q F_V^T) F_V for each of the F frames, the softmax over the
+    frame's N tokens, unscaled scores.  query_bits bf16 bits [C][d],
+    feature_bits bf16 bits [F][N][d] (uint16).  Returns [F][C][d] float64."""
+    lib = _load()
+    q = _c(query_bits, np.uint16)
+    f = _c(feature_bits, np.uint16)
+    if f.ndim == 2:
+        f = f[None]
+    C, d = q.shape
+    F, N, d2 = f.shape
+    assert d2 == d
+    out = np.zeros((F, C, d), np.float64)
+    st = lib.oracle_visual_compress(_ptr(q), _ptr(f), F, N, C, d, _ptr(out))
+    if st != ORACLE_OK:
+        raise OracleError(f"oracle_visual_compress status {st}")
+    return out
 
 
 def _bf16_to_f64(bits):

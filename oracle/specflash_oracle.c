@@ -33,6 +33,10 @@
  *      were accepted.  At temperature 0 (greedy decoding, Sec. 4.2) a draft is
  *      accepted iff it equals the argmax of the target logits.
  *
+ *   4. KV commit after acceptance, draft-tail sampling (Algorithm 1) and
+ *      visual token compression (Sec. 3.2, Eq. 3), each described at its
+ *      function below.
+ *
  * Readings of points the paper leaves open (each one is listed with its
  * reason in the design notes of the repository):
  *   - acceptance test: u * q(x) < p(x) with a strict "<" (u in [0,1));
@@ -559,5 +563,62 @@ int oracle_sample(const float *logits, const float *uniforms, const float *tempe
         if (margin)
             margin[r] = nearest;
     }
+    return ORACLE_OK;
+}
+
+/* ------------------------------------------------------------------------ */
+/* Visual token compression (Sec. 3.2, Eq. 3; Algorithm 1): the draft model */
+/* compresses the N visual features F_V of an image or frame into C          */
+/* features with a learnable query set Q (C x d):                             */
+/*     F^_V = softmax(Q F_V^T) F_V,                                           */
+/* F_V serving as both keys and values.  Readings: the softmax runs over the */
+/* N visual tokens of one query (its weights sum to 1), the scores are not   */
+/* scaled (Eq. 3 writes none), and a clip of F frames is F independent        */
+/* images of N tokens each sharing the same queries.                          */
+/*                                                                            */
+/* queries   bf16 bits [C][d]                                                 */
+/* features  bf16 bits [F][N][d]                                              */
+/* out       [F][C][d] doubles                                                */
+/* ------------------------------------------------------------------------ */
+int oracle_visual_compress(const uint16_t *queries, const uint16_t *features, int F, int N, int C,
+                           int d, double *out)
+{
+    if (F < 1 || N < 1 || C < 1 || d < 1)
+        return ORACLE_ERR_ARG;
+    double *s = (double *)malloc(sizeof(double) * (size_t)N);
+    if (!s)
+        return ORACLE_ERR_NOMEM;
+    for (int f = 0; f < F; ++f) {
+        const uint16_t *fv = features + (size_t)f * N * d;
+        for (int c = 0; c < C; ++c) {
+            const uint16_t *qc = queries + (size_t)c * d;
+            /* scores of query c against every token of the frame */
+            double smax = -INFINITY;
+            for (int n = 0; n < N; ++n) {
+                double acc = 0.0;
+                for (int j = 0; j < d; ++j)
+                    acc += oracle_bf16_value(qc[j]) * oracle_bf16_value(fv[(size_t)n * d + j]);
+                s[n] = acc;
+                if (acc > smax)
+                    smax = acc;
+            }
+            /* softmax over the tokens */
+            double z = 0.0;
+            for (int n = 0; n < N; ++n) {
+                s[n] = exp(s[n] - smax);
+                z += s[n];
+            }
+            /* weighted sum of the token features */
+            double *o = out + ((size_t)f * C + c) * d;
+            for (int j = 0; j < d; ++j)
+                o[j] = 0.0;
+            for (int n = 0; n < N; ++n) {
+                const double w = s[n] / z;
+                for (int j = 0; j < d; ++j)
+                    o[j] += w * oracle_bf16_value(fv[(size_t)n * d + j]);
+            }
+        }
+    }
+    free(s);
     return ORACLE_OK;
 }

@@ -58,6 +58,18 @@ MUTANTS = {
     "sample_greedy_last_max": ("        for (int x = 1; x < V; ++x)\n            if (row[x] > row[best])\n                best = x;",
                                "        for (int x = 1; x < V; ++x)\n            if (row[x] >= row[best])\n                best = x;"),
     "sample_unnormalised_probs": ("            pr[x] /= S;", "            pr[x] /= 1.0;"),
+    "compress_scaled_scores": ("                s[n] = acc;\n                if (acc > smax)",
+                               "                s[n] = acc / sqrt((double)d);\n                if (acc > smax)"),
+    "compress_every_frame_reads_frame_zero": ("        const uint16_t *fv = features + (size_t)f * N * d;",
+                                              "        const uint16_t *fv = features;"),
+    "compress_weights_not_normalised": ("                const double w = s[n] / z;",
+                                        "                const double w = s[n] / (double)N;"),
+    "compress_negated_exponent": ("                s[n] = exp(s[n] - smax);",
+                                  "                s[n] = exp(smax - s[n]);"),
+    "compress_values_from_queries": ("                    o[j] += w * oracle_bf16_value(fv[(size_t)n * d + j]);",
+                                     "                    o[j] += w * oracle_bf16_value(qc[j]);"),
+    "compress_scores_skip_last_column": ("                for (int j = 0; j < d; ++j)\n                    acc +=",
+                                         "                for (int j = 0; j < d - 1; ++j)\n                    acc +="),
 }
 
 
@@ -86,6 +98,7 @@ def test_pins_reject_mutant(name, source, tmp_path):
          os.path.join(ROOT, "tests", "test_oracle_attention.py"),
          os.path.join(ROOT, "tests", "test_oracle_accept.py"),
          os.path.join(ROOT, "tests", "test_oracle_kv_commit.py"),
-         os.path.join(ROOT, "tests", "test_oracle_sample.py")],
+         os.path.join(ROOT, "tests", "test_oracle_sample.py"),
+         os.path.join(ROOT, "tests", "test_oracle_compress.py")],
         cwd=ROOT, env=env, capture_output=True, text=True, timeout=600)
     assert proc.returncode != 0, f"mutant {name} survived the oracle pins:\n{proc.stdout[-2000:]}"
