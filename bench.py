@@ -344,6 +344,55 @@ def time_draft_tail(wl, dev, stream, capture):
             "probs_sum_to_one": ok, "device_status": status}
 
 
+def time_visual_compress(wl, dev, stream, capture):
+    """Device time of sf_visual_compress (the draft model's Eq. 3 compressor)
+    over the workload's frames, and of its score projection alone
+    (sf_lm_head with the queries as rows and the features as the weight
+    matrix), each replayed from a CUDA graph of 10 calls."""
+    import torch
+    from paper_2505_12728_gb300 import specflash_verify as sfv
+    from paper_2505_12728_gb300.workloads import COMPRESS_SHAPES, make_compress_inputs
+    if wl.name not in COMPRESS_SHAPES:
+        return None
+    F, N, C, d = COMPRESS_SHAPES[wl.name]
+    qb, fb = make_compress_inputs(wl)
+    bf = lambda bits: torch.from_numpy(np.ascontiguousarray(bits).view(np.int16)).to(dev).view(
+        torch.bfloat16)
+    q, f = bf(qb), bf(fb)
+    out = torch.empty((F, C, d), dtype=torch.bfloat16, device=dev)
+    ws = sfv.new_workspace(sfv.visual_compress_workspace_size(F, N, C), dev)
+    scores = torch.empty((C, F * N), dtype=torch.float32, device=dev)
+    ws2 = sfv.new_workspace(sfv.draft_tail_workspace_size(C, F * N), dev)
+    full = lambda: sfv.visual_compress(q, f, out=out, workspace=ws, stream=stream)
+    proj = lambda: sfv.lm_head(q, f.view(F * N, d), logits=scores, workspace=ws2, stream=stream)
+
+    def per_call_us(fn, calls=10, reps=5):
+        fn()
+        g = capture(lambda: [fn() for _ in range(calls)])
+        g.replay()
+        a = torch.cuda.Event(enable_timing=True)
+        b = torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        for _ in range(reps):
+            g.replay()
+        b.record(stream)
+        torch.cuda.synchronize()
+        return a.elapsed_time(b) * 1e3 / (calls * reps)
+
+    full_us = per_call_us(full)
+    proj_us = per_call_us(proj)
+    peak, kind = measured_peaks()
+    alg = F * N * d * 2 + C * d * 2 + F * C * d * 2  # features once, queries, output
+    flops = 4.0 * F * C * N * d
+    return {"frames": F, "tokens_per_frame": N, "queries": C, "hidden": d,
+            "visual_compress_us": full_us, "scores_projection_us": proj_us,
+            "gbs": alg / (full_us * 1e-6) / 1e9, "frac": alg / (full_us * 1e-6) / 1e9 / peak,
+            "tflops": flops / (full_us * 1e-6) / 1e12, "algorithmic_bytes": alg,
+            "peak_gbs": peak, "peak_source": kind,
+            "kernels": ["lm_head_kernel", "compress_apply_kernel"],
+            "device_status": sfv.read_device_status(ws)}
+
+
 def workload_config(wl, seq_lens):
     return {"workload": wl.name, "description": wl.description, "batch": wl.B,
             "layers": wl.layers, "H_q": wl.H_q, "H_kv": wl.H_kv, "head_dim": wl.d,
@@ -510,6 +559,7 @@ def run_ours(args):
     # ---- draft-distribution tail (the LM head, softmax and sampling of the
     # B*k draft rows that produce q and T'; outside the verification step)
     dt = time_draft_tail(wl, dev, stream, capture) if not args.no_draft_tail else None
+    vcomp = time_visual_compress(wl, dev, stream, capture) if not args.no_draft_tail else None
 
     # ---- end to end through host buffers ----
     pin = lambda a: torch.from_numpy(np.ascontiguousarray(a)).pin_memory()
@@ -577,6 +627,7 @@ def run_ours(args):
         "accept_gbs": accept_bytes(wl, sampling_rows) / (acc_launch_ms / 1e3) / 1e9,
         "kv_commit_us": commit_us,
         "draft_tail": dt,
+        "visual_compress": vcomp,
         "mean_accepted": float(n_acc.float().mean().item()),
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                      "frac": achieved / peak,
@@ -618,7 +669,7 @@ def main(argv=None):
                     help="seconds of oracle work for the cpu_baseline sample")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-draft-tail", action="store_true",
-                    help="skip the draft-tail (LM head + sampling) timing")
+                    help="skip the draft-side timings (LM head + sampling, visual compressor)")
     ap.add_argument("--eager", action="store_true",
                     help="launch every call from Python instead of replaying CUDA graphs")
     args = ap.parse_args(argv)

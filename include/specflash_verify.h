@@ -299,6 +299,31 @@ int sf_draft_sample(const void *hidden, const void *weight, const float *uniform
                     float *probs, int32_t *tokens, void *workspace, size_t workspace_bytes,
                     cudaStream_t stream);
 
+/* ------------------------------------------------------------------------ */
+/* Visual token compression of the draft model (Sec. 3.2, Eq. 3; Algorithm */
+/* 1): each image or video frame's N visual features F_V (the target's      */
+/* second-to-top layer) are compressed to C features with the learnable     */
+/* query set Q, F_V serving as keys and values:                             */
+/*     out[f] = softmax(Q F_V[f]^T) F_V[f],                                 */
+/* the softmax over the frame's N tokens for each query, scores unscaled.  */
+/*                                                                           */
+/* queries   bf16 [C][d], 16-byte aligned.                                  */
+/* features  bf16 [F][N][d], 16-byte aligned.                               */
+/* out       bf16 [F][C][d], 16-byte aligned.                               */
+/* Limits: 1 <= F <= 65535, 1 <= N <= 768, 1 <= C <= 128, d a multiple of   */
+/* 128 in [128, 2^20], F * N <= SF_MAX_VOCAB.                               */
+/* workspace >= sf_visual_compress_workspace_size(F, N, C) bytes (it holds  */
+/*           the fp32 scores), 256-byte aligned, zero-filled before first    */
+/*           use (status word).                                              */
+/* Two launches; both copy their inputs only after the previous kernel on   */
+/* the stream completes.  Deterministic; SF_DEVICE_TIMEOUT is the only      */
+/* device status.                                                            */
+/* ------------------------------------------------------------------------ */
+size_t sf_visual_compress_workspace_size(int F, int N, int C);
+
+int sf_visual_compress(const void *queries, const void *features, int F, int N, int C, int d,
+                       void *out, void *workspace, size_t workspace_bytes, cudaStream_t stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -89,6 +89,8 @@ struct LmParams {
   uint32_t stage_bytes;  // weight box + NP * 128 bytes of hidden states
   uint32_t tmem_cols;
   uint32_t idesc;
+  int w_after_wait;  // copy the weight rows only after griddepcontrol.wait
+  int w_keep;        // weight rows are re-read next: L2 evict_last instead of evict_first
 };
 
 struct SampleParams {
@@ -199,11 +201,12 @@ lm_head_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
 
   if (warp == kLmProducerWarp) {
     if (lane == 0) {
-      const uint64_t pol_w = l2_policy_evict_first();
+      const uint64_t pol_w = p.w_keep ? l2_policy_evict_last() : l2_policy_evict_first();
       const uint64_t pol_h = l2_policy_evict_last();
       const uint32_t prime = total < static_cast<uint32_t>(S) ? total : static_cast<uint32_t>(S);
-      // the first ring fill: weights before the dependency wait, hidden
-      // states (possibly written by the previous kernel) after it
+      // the first ring fill: weights before the dependency wait (unless
+      // they may come from the previous kernel), hidden states after it
+      if (p.w_after_wait) grid_dependency_wait();
       for (uint32_t q = 0; q < prime; ++q) {
         const int i = static_cast<int>(q) / p.KC, kc = static_cast<int>(q) % p.KC;
         uint32_t bytes;
@@ -212,7 +215,7 @@ lm_head_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
         tma_load_2d(ring + q * p.stage_bytes, mw, kc * kLmChunkK, v0 + i * kLmTileV, bar(FULL + q),
                     pol_w);
       }
-      grid_dependency_wait();
+      if (!p.w_after_wait) grid_dependency_wait();
       for (uint32_t q = 0; q < prime; ++q) {
         const int kc = static_cast<int>(q) % p.KC;
         tma_load_2d(ring + q * p.stage_bytes + kLmWBytes, &tmap_h, kc * kLmChunkK, 0, bar(FULL + q),
@@ -697,7 +700,8 @@ static cudaLaunchConfig_t pdl_config(dim3 grid, dim3 block, size_t smem, cudaStr
 // sampling statistics [R][G] and *G_out receives G.
 static int launch_lm_head(const void *hidden, const void *weight, int R, int hidden_size, int V,
                           float *logits, const float *temperature, SampStat *stats, uint32_t *status,
-                          int *G_out, cudaStream_t stream) {
+                          int *G_out, cudaStream_t stream, bool w_after_wait = false,
+                          bool w_keep = false) {
   DeviceInfo dev;
   int st = current_device(&dev);
   if (st != SF_OK) return st;
@@ -725,6 +729,8 @@ static int launch_lm_head(const void *hidden, const void *weight, int R, int hid
   while (cols < 2u * static_cast<uint32_t>(NP)) cols <<= 1;
   prm.tmem_cols = cols;
   prm.idesc = idesc_bf16_f32(128, NP, 0, 0);
+  prm.w_after_wait = w_after_wait ? 1 : 0;
+  prm.w_keep = w_keep ? 1 : 0;
   const size_t smem = LmSmem::bytes(prm.stages, prm.stage_bytes, NP);
   if (smem > static_cast<size_t>(dev.max_smem_optin))
     return fail(SF_ERR_UNSUPPORTED, "LM-head ring needs %zu bytes of shared memory", smem);
@@ -766,6 +772,15 @@ static int launch_finish(SampleParams prm, cudaStream_t stream) {
   cudaError_t e = cudaLaunchKernelEx(&cfg, sample_finish_kernel, prm);
   if (e != cudaSuccess) return fail(SF_ERR_CUDA, "sampling launch: %s", cudaGetErrorString(e));
   return SF_OK;
+}
+
+int launch_projection(const void *rows_r, const void *rows_v, int R, int hidden_size, int V,
+                      float *out, uint32_t *status, bool inputs_after_wait, bool keep_v_rows,
+                      cudaStream_t stream) {
+  const int st = check_lm_args(rows_r, rows_v, R, hidden_size, V, out);
+  if (st != SF_OK) return st;
+  return launch_lm_head(rows_r, rows_v, R, hidden_size, V, out, nullptr, nullptr, status, nullptr,
+                        stream, inputs_after_wait, keep_v_rows);
 }
 
 }  // namespace sf

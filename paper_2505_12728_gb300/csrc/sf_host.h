@@ -31,6 +31,14 @@ int current_device(DeviceInfo *info);
 int encode_tensor_map_bf16(CUtensorMap *map, const void *base, int rank, const uint64_t *dims,
                            const uint64_t *strides, const uint32_t *box);
 
+// out[r][v] = sum_j rows_r[r][j] * rows_v[v][j] (bf16 in, fp32 out) with the
+// tcgen05 projection kernel of draft_tail.cu (1 <= R <= 256).  With
+// inputs_after_wait both inputs are copied only after the previous kernel on
+// the stream completes; keep_v_rows leaves rows_v in L2 for a second pass.
+int launch_projection(const void *rows_r, const void *rows_v, int R, int hidden_size, int V,
+                      float *out, uint32_t *status, bool inputs_after_wait, bool keep_v_rows,
+                      cudaStream_t stream);
+
 inline bool aligned(const void *p, size_t a) {
   return (reinterpret_cast<uintptr_t>(p) % a) == 0;
 }

@@ -32,6 +32,7 @@ EXPORTED_SYMBOLS = (
     "sf_accept_workspace_size", "sf_accept",
     "sf_kv_commit_workspace_size", "sf_kv_commit",
     "sf_draft_tail_workspace_size", "sf_lm_head", "sf_sample", "sf_draft_sample",
+    "sf_visual_compress_workspace_size", "sf_visual_compress",
 )
 
 _lock = threading.Lock()
@@ -96,6 +97,10 @@ def load_library(path: str | None = None):
         lib.sf_sample.restype = I
         lib.sf_draft_sample.argtypes = [P, P, P, P, I, I, I, P, P, P, P, S, P]
         lib.sf_draft_sample.restype = I
+        lib.sf_visual_compress_workspace_size.argtypes = [I, I, I]
+        lib.sf_visual_compress_workspace_size.restype = S
+        lib.sf_visual_compress.argtypes = [P, P, I, I, I, I, P, P, S, P]
+        lib.sf_visual_compress.restype = I
         _lib = lib
         return lib
 
@@ -369,3 +374,33 @@ def draft_sample(hidden, weight, uniforms, temperature, *, logits=None, probs=No
         _ptr(hidden), _ptr(weight), _ptr(uniforms), _ptr(temperature), R, Hd, V, _ptr(logits),
         _ptr(probs), _ptr(tokens), _ptr(workspace), workspace.numel(), _stream_handle(stream)))
     return logits, probs, tokens
+
+
+# --------------------------------------------------------------------------- #
+# visual token compression                                                    #
+# --------------------------------------------------------------------------- #
+def visual_compress_workspace_size(F, N, C) -> int:
+    n = load_library().sf_visual_compress_workspace_size(F, N, C)
+    if n == 0:
+        raise SFError(1, "invalid compressor shape")
+    return int(n)
+
+
+def visual_compress(queries, features, *, out=None, workspace=None, stream=None):
+    """sf_visual_compress: queries bf16 [C][d], features bf16 [F][N][d].
+    Returns out bf16 [F][C][d] = softmax(Q F_V^T) F_V per frame."""
+    C, d = queries.shape
+    F, N, d2 = features.shape
+    _need(queries, "queries", torch.bfloat16)
+    _need(features, "features", torch.bfloat16)
+    if d2 != d:
+        raise ValueError("queries and features differ in d")
+    if out is None:
+        out = torch.empty((F, C, d), dtype=torch.bfloat16, device=queries.device)
+    _need(out, "out", torch.bfloat16, (F, C, d))
+    if workspace is None:
+        workspace = new_workspace(visual_compress_workspace_size(F, N, C), queries.device)
+    _check(load_library().sf_visual_compress(_ptr(queries), _ptr(features), F, N, C, d, _ptr(out),
+                                             _ptr(workspace), workspace.numel(),
+                                             _stream_handle(stream)))
+    return out

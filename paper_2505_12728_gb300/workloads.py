@@ -334,3 +334,33 @@ def make_sample_case(R, V, seed, temperature=None, logit_std=3.0):
     if temperature is None:
         temperature = np.ones(R, np.float32)
     return logits, uniforms, np.asarray(temperature, np.float32).reshape(R)
+
+
+
+# --------------------------------------------------------------------------- #
+# visual-compressor inputs                                                    #
+# --------------------------------------------------------------------------- #
+# (frames F, tokens per frame N, queries C, hidden d) per workload, at the
+# paper's compression ratio C/N = 1/9: LLaVA images 576 -> 64 (d 4096), QwenVL
+# images 324 -> 36 and video frames 144 -> 16 (d 3584).
+COMPRESS_SHAPES = {
+    "tiny": (1, 576, 64, 4096),
+    "image7b": (5, 576, 64, 4096),     # the 5 images of the image7b prefix
+    "gqa": (8, 324, 36, 3584),         # one QwenVL image per sequence
+    "video": (128, 144, 16, 3584),     # 4 sequences x 32 frames
+}
+
+
+def make_compress_case(F, N, C, d, seed, q_std=2.0):
+    """Features F_V ~ N(0, 1) [F][N][d] and queries ~ N(0, q_std^2 / d)
+    [C][d], both bf16 bits, so the scores are ~ N(0, q_std^2)."""
+    rng = np.random.default_rng(seed)
+    queries = _scaled_normal_bf16(rng, (C, d), q_std / np.sqrt(d))
+    features = _normal_bf16(rng, (F, N, d))
+    return queries, features
+
+
+def make_compress_inputs(wl: Workload, seed=None):
+    seed = wl.seed if seed is None else seed
+    F, N, C, d = COMPRESS_SHAPES[wl.name]
+    return make_compress_case(F, N, C, d, seed=[seed, 0xC0C0])
