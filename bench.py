@@ -360,7 +360,7 @@ def time_visual_compress(wl, dev, stream, capture):
         torch.bfloat16)
     q, f = bf(qb), bf(fb)
     out = torch.empty((F, C, d), dtype=torch.bfloat16, device=dev)
-    ws = sfv.new_workspace(sfv.visual_compress_workspace_size(F, N, C), dev)
+    ws = sfv.new_workspace(sfv.visual_compress_workspace_size(F, N, C, d), dev)
     scores = torch.empty((C, F * N), dtype=torch.float32, device=dev)
     ws2 = sfv.new_workspace(sfv.draft_tail_workspace_size(C, F * N), dev)
     full = lambda: sfv.visual_compress(q, f, out=out, workspace=ws, stream=stream)

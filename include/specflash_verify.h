@@ -312,14 +312,14 @@ int sf_draft_sample(const void *hidden, const void *weight, const float *uniform
 /* out       bf16 [F][C][d], 16-byte aligned.                               */
 /* Limits: 1 <= F <= 65535, 1 <= N <= 768, 1 <= C <= 128, d a multiple of   */
 /* 128 in [128, 2^20], F * N <= SF_MAX_VOCAB.                               */
-/* workspace >= sf_visual_compress_workspace_size(F, N, C) bytes (it holds  */
-/*           the fp32 scores), 256-byte aligned, zero-filled before first    */
-/*           use (status word).                                              */
-/* Two launches; both copy their inputs only after the previous kernel on   */
+/* workspace >= sf_visual_compress_workspace_size(F, N, C, d) bytes (fp32  */
+/*           partial scores, bf16 weights, their sums), 256-byte aligned,   */
+/*           zero-filled before first use (status word).                    */
+/* Three launches; each copies its inputs only after the previous kernel on */
 /* the stream completes.  Deterministic; SF_DEVICE_TIMEOUT is the only      */
 /* device status.                                                            */
 /* ------------------------------------------------------------------------ */
-size_t sf_visual_compress_workspace_size(int F, int N, int C);
+size_t sf_visual_compress_workspace_size(int F, int N, int C, int d);
 
 int sf_visual_compress(const void *queries, const void *features, int F, int N, int C, int d,
                        void *out, void *workspace, size_t workspace_bytes, cudaStream_t stream);

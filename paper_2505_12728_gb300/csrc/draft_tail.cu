@@ -91,6 +91,8 @@ struct LmParams {
   uint32_t idesc;
   int w_after_wait;  // copy the weight rows only after griddepcontrol.wait
   int w_keep;        // weight rows are re-read next: L2 evict_last instead of evict_first
+  int ks;            // hidden-dimension splits: CTA (g, s) sums chunks [s*KC/ks, (s+1)*KC/ks)
+  long long part_stride;  // floats between the ks partial outputs (split s adds s * part_stride)
 };
 
 struct SampleParams {
@@ -158,11 +160,15 @@ lm_head_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
   auto bar = [&](int i) -> uint32_t { return bars + 8u * static_cast<uint32_t>(i); };
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int v0 = static_cast<int>(static_cast<long long>(blockIdx.x) * p.V / p.G);
-  const int v1 = static_cast<int>(static_cast<long long>(blockIdx.x + 1) * p.V / p.G);
+  const int grp = static_cast<int>(blockIdx.x) % p.G, split = static_cast<int>(blockIdx.x) / p.G;
+  const int v0 = static_cast<int>(static_cast<long long>(grp) * p.V / p.G);
+  const int v1 = static_cast<int>(static_cast<long long>(grp + 1) * p.V / p.G);
   const int n_tiles = (v1 - v0 + kLmTileV - 1) / kLmTileV;
   const int last_h = v1 - v0 - (n_tiles - 1) * kLmTileV;  // rows of the last tile
-  const uint32_t total = static_cast<uint32_t>(n_tiles) * static_cast<uint32_t>(p.KC);
+  const int kc0 = split * p.KC / p.ks;                      // this CTA's hidden chunks
+  const int nkc = (split + 1) * p.KC / p.ks - kc0;
+  float *const logits = p.logits + static_cast<long long>(split) * p.part_stride;
+  const uint32_t total = static_cast<uint32_t>(n_tiles) * static_cast<uint32_t>(nkc);
   // weight map and box height of tile i
   auto tile_map = [&](int i, uint32_t &bytes) -> const CUtensorMap * {
     const int h = i == n_tiles - 1 ? last_h : kLmTileV;
@@ -208,7 +214,7 @@ lm_head_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
       // they may come from the previous kernel), hidden states after it
       if (p.w_after_wait) grid_dependency_wait();
       for (uint32_t q = 0; q < prime; ++q) {
-        const int i = static_cast<int>(q) / p.KC, kc = static_cast<int>(q) % p.KC;
+        const int i = static_cast<int>(q) / nkc, kc = kc0 + static_cast<int>(q) % nkc;
         uint32_t bytes;
         const CUtensorMap *mw = tile_map(i, bytes);
         mbar_arrive_expect_tx(bar(FULL + q), bytes);
@@ -217,7 +223,7 @@ lm_head_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
       }
       if (!p.w_after_wait) grid_dependency_wait();
       for (uint32_t q = 0; q < prime; ++q) {
-        const int kc = static_cast<int>(q) % p.KC;
+        const int kc = kc0 + static_cast<int>(q) % nkc;
         tma_load_2d(ring + q * p.stage_bytes + kLmWBytes, &tmap_h, kc * kLmChunkK, 0, bar(FULL + q),
                     pol_h);
       }
@@ -225,7 +231,7 @@ lm_head_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
       for (; q < total; ++q) {
         const uint32_t slot = q % S;
         if (!mbar_wait_or_abort(bar(EMPTY + slot), ((q / S) - 1) & 1u, s_abort)) break;
-        const int i = static_cast<int>(q / p.KC), kc = static_cast<int>(q % p.KC);
+        const int i = static_cast<int>(q) / nkc, kc = kc0 + static_cast<int>(q) % nkc;
         const uint32_t dst = ring + slot * p.stage_bytes;
         uint32_t bytes;
         const CUtensorMap *mw = tile_map(i, bytes);
@@ -254,7 +260,7 @@ lm_head_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
       }
       tc_fence_after_sync();
       const uint32_t d = tmem + buf * static_cast<uint32_t>(p.NP);
-      for (int kc = 0; kc < p.KC; ++kc, ++q) {
+      for (int kc = 0; kc < nkc; ++kc, ++q) {
         const uint32_t slot = q % S;
         int w = 1;
         if (lane == 0) w = mbar_wait_or_abort(bar(FULL + slot), (q / S) & 1u, s_abort);
@@ -318,7 +324,7 @@ lm_head_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
         if (vin) {
 #pragma unroll
           for (int j = 0; j < 16; ++j)
-            if (c0 + j < p.R) p.logits[static_cast<size_t>(c0 + j) * p.V + v] = __uint_as_float(x[j]);
+            if (c0 + j < p.R) logits[static_cast<size_t>(c0 + j) * p.V + v] = __uint_as_float(x[j]);
         }
         if (!stats) continue;
         float *tb = tbuf + (g_count & 1u) * (kLmColGroup * kLmTStride);
@@ -364,7 +370,7 @@ lm_head_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
     if (stats) {
       named_bar_sync(1, kLmEpiThreads);
       for (int c = tid; c < p.R; c += kLmEpiThreads)
-        p.stats[static_cast<size_t>(c) * p.G + blockIdx.x] = run[c];
+        p.stats[static_cast<size_t>(c) * p.G + grp] = run[c];
     }
   }
 
@@ -701,7 +707,7 @@ static cudaLaunchConfig_t pdl_config(dim3 grid, dim3 block, size_t smem, cudaStr
 static int launch_lm_head(const void *hidden, const void *weight, int R, int hidden_size, int V,
                           float *logits, const float *temperature, SampStat *stats, uint32_t *status,
                           int *G_out, cudaStream_t stream, bool w_after_wait = false,
-                          bool w_keep = false) {
+                          bool w_keep = false, int ks = 1) {
   DeviceInfo dev;
   int st = current_device(&dev);
   if (st != SF_OK) return st;
@@ -731,6 +737,9 @@ static int launch_lm_head(const void *hidden, const void *weight, int R, int hid
   prm.idesc = idesc_bf16_f32(128, NP, 0, 0);
   prm.w_after_wait = w_after_wait ? 1 : 0;
   prm.w_keep = w_keep ? 1 : 0;
+  prm.ks = ks < 1 ? 1 : (ks > prm.KC ? prm.KC : ks);
+  prm.part_stride = static_cast<long long>(R) * V;
+  if (stats && prm.ks != 1) return fail(SF_ERR_INVALID_ARG, "statistics need an unsplit projection");
   const size_t smem = LmSmem::bytes(prm.stages, prm.stage_bytes, NP);
   if (smem > static_cast<size_t>(dev.max_smem_optin))
     return fail(SF_ERR_UNSUPPORTED, "LM-head ring needs %zu bytes of shared memory", smem);
@@ -744,7 +753,7 @@ static int launch_lm_head(const void *hidden, const void *weight, int R, int hid
   st = lm_tensor_map(&th, hidden, static_cast<uint64_t>(R), hidden_size, static_cast<uint32_t>(NP));
   if (st != SF_OK) return st;
   cudaLaunchAttribute attr[1];
-  cudaLaunchConfig_t cfg = pdl_config(dim3(prm.G), dim3(kLmThreads), smem, stream, attr);
+  cudaLaunchConfig_t cfg = pdl_config(dim3(prm.G * prm.ks), dim3(kLmThreads), smem, stream, attr);
   cudaError_t e = cudaLaunchKernelEx(&cfg, lm_head_kernel, tw, twa, twb, th, prm);
   if (e != cudaSuccess) return fail(SF_ERR_CUDA, "LM-head launch: %s", cudaGetErrorString(e));
   if (G_out) *G_out = prm.G;
@@ -774,13 +783,22 @@ static int launch_finish(SampleParams prm, cudaStream_t stream) {
   return SF_OK;
 }
 
+int projection_splits(int V, int hidden_size, int sm_count) {
+  const int tiles = (V + kLmTileV - 1) / kLmTileV;
+  const int G = tiles < sm_count ? tiles : sm_count;
+  const int KC = (hidden_size + kLmChunkK - 1) / kLmChunkK;
+  int ks = sm_count / G;
+  if (ks > KC) ks = KC;
+  return ks < 1 ? 1 : ks;
+}
+
 int launch_projection(const void *rows_r, const void *rows_v, int R, int hidden_size, int V,
                       float *out, uint32_t *status, bool inputs_after_wait, bool keep_v_rows,
-                      cudaStream_t stream) {
+                      int splits, cudaStream_t stream) {
   const int st = check_lm_args(rows_r, rows_v, R, hidden_size, V, out);
   if (st != SF_OK) return st;
   return launch_lm_head(rows_r, rows_v, R, hidden_size, V, out, nullptr, nullptr, status, nullptr,
-                        stream, inputs_after_wait, keep_v_rows);
+                        stream, inputs_after_wait, keep_v_rows, splits);
 }
 
 }  // namespace sf

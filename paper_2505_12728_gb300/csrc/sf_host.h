@@ -35,9 +35,14 @@ int encode_tensor_map_bf16(CUtensorMap *map, const void *base, int rank, const u
 // tcgen05 projection kernel of draft_tail.cu (1 <= R <= 256).  With
 // inputs_after_wait both inputs are copied only after the previous kernel on
 // the stream completes; keep_v_rows leaves rows_v in L2 for a second pass.
+// With splits > 1 the hidden dimension is cut into `splits` ranges and
+// split s writes its partial sums to out + s * R * V (the caller adds them).
 int launch_projection(const void *rows_r, const void *rows_v, int R, int hidden_size, int V,
                       float *out, uint32_t *status, bool inputs_after_wait, bool keep_v_rows,
-                      cudaStream_t stream);
+                      int splits, cudaStream_t stream);
+
+// Hidden-dimension splits that fill the GPU when V has few 128-row tiles.
+int projection_splits(int V, int hidden_size, int sm_count);
 
 inline bool aligned(const void *p, size_t a) {
   return (reinterpret_cast<uintptr_t>(p) % a) == 0;

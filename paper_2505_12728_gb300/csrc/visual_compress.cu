@@ -12,21 +12,26 @@
 // GB300 design.  The work is 4 C N d flops per frame over 2 N d bytes of
 // features: 2 C = 128 flop/byte for LLaVA, below the bf16 tensor ridge
 // (~286), so the floor is reading the features once at HBM speed, and only
-// tensor cores keep the arithmetic under that.  Two launches:
+// tensor cores keep the arithmetic under that.  Three launches:
 //  1. scores S = Q F_V^T for all frames at once ([C][F*N] fp32) with the
-//     tcgen05 projection kernel of draft_tail.cu (queries as the N side,
-//     the F*N feature rows streamed as the M side); it copies the features
-//     after the dependency wait and leaves them in L2 (evict_last) for 2.;
-//  2. compress_apply_kernel, one CTA per (128 output columns, frame): warp 5
-//     copies the frame's features for those columns into shared memory
-//     ([64-column half][N tokens][128 B], 128B-swizzled: the MN-major B
-//     operand); warps 0-3 hold one query per TMEM lane, read its N scores,
-//     and store the unnormalised weights exp(s - max) as bf16 into tensor
-//     memory (the A operand); warp 4 issues O = P F_V as N/16 MMAs of M = 128
-//     (queries), N = 128 (columns), K = 16 (tokens); warps 0-3 divide by the
-//     sum of the bf16 weights and store bf16 rows.
-// N is at most 768 (P takes N/2 TMEM columns beside the 128 of O) and C at
-// most 128 (one lane per query).  Every wait is bounded (SF_DEVICE_TIMEOUT).
+//     tcgen05 projection kernel of draft_tail.cu (queries as the N side, the
+//     F*N feature rows streamed as the M side), the hidden dimension split
+//     into ks ranges when F*N has too few 128-row tiles to fill the GPU
+//     (each split writes partial sums); it copies the features after the
+//     dependency wait and leaves them in L2 (evict_last) for 3.;
+//  2. compress_softmax_kernel: one warp per (frame, query) sums the ks
+//     partials in a fixed order, takes the row max, and writes the
+//     unnormalised weights exp(s - max) rounded to bf16 into P [C][F][Np]
+//     (Np = N rounded up to 64, zeros past N) and the sum of the rounded
+//     weights into l [F][C];
+//  3. compress_apply_kernel, one CTA per (128 output columns, frame): the
+//     transposed product O^T = F_V^T P^T as a pipelined tcgen05 GEMM with
+//     M = 128 feature columns (A = the frame's features, MN-major, two
+//     64-column boxes per 64 tokens), N = C padded to 16 (B = P, K-major) and
+//     K = 64 tokens per ring slot, the accumulator in tensor memory; warps 0-3
+//     (lane = feature column) divide by l and store bf16, coalesced along d.
+// N is at most 768 and C at most 128.  Every wait is bounded
+// (SF_DEVICE_TIMEOUT).
 #include <cmath>
 #include <mutex>
 
@@ -38,54 +43,121 @@ namespace sf {
 constexpr int kVcThreads = 192;
 constexpr int kVcMmaWarp = 4;
 constexpr int kVcProducerWarp = 5;
-constexpr int kVcCols = 128;        // output columns per CTA (MMA N)
+constexpr int kVcCols = 128;        // output columns per CTA (MMA M)
+constexpr int kVcTokens = 64;       // tokens per ring slot (K)
 constexpr int kVcMaxTokens = 768;   // N
 constexpr int kVcMaxQueries = 128;  // C
-constexpr uint32_t kVcTmemCols = 512;
-constexpr uint32_t kVcTmemO = 0, kVcTmemP = 128;
+constexpr int kVcMaxStages = 4;
+constexpr uint32_t kVcFBytes = 2 * kVcTokens * 128;  // 64 tokens x 128 columns of features
+constexpr int kVcSoftmaxWarps = 8;
 
-struct VcParams {
-  const float *scores;  // [C][F*N]
-  __nv_bfloat16 *out;   // [F][C][d]
-  uint32_t *status;
-  long long score_stride;  // F*N
-  int F, N, C, d;
-  int Npad;             // N rounded up to 16 (MMA K)
-  int BT;               // token rows per TMA box (divides Npad)
-  int vec4;             // score rows are 16-byte aligned (N % 4 == 0)
+struct VcSoftmaxParams {
+  const float *scores;  // [ks][C][F*N]
+  __nv_bfloat16 *P;     // [C][F*Np]
+  float *l;             // [F][C]
+  long long part_stride;  // C*F*N
+  int ks, F, N, C, Np;
 };
 
-static size_t vc_smem_bytes(int Npad) {
-  return 1024 + 2 * static_cast<size_t>(Npad) * 128 + 64;
+struct VcParams {
+  const float *l;       // [F][C]
+  __nv_bfloat16 *out;   // [F][C][d]
+  uint32_t *status;
+  int F, N, C, Cp, d, Np;
+  int KT;               // Np / 64 ring slots per CTA
+  int stages;
+  uint32_t stage_bytes;
+  uint32_t tmem_cols;
+};
+
+static size_t vc_smem_bytes(int stages, uint32_t stage_bytes, int C) {
+  return 1024 + static_cast<size_t>(stages) * stage_bytes + 8 * (2 * stages + 1) + 64 + 4 * C;
+}
+
+// grid (F, ceil(C / 8)), 256 threads: warp w handles query 8 * blockIdx.y + w
+// of frame blockIdx.x.
+__global__ void __launch_bounds__(32 * kVcSoftmaxWarps)
+compress_softmax_kernel(const __grid_constant__ VcSoftmaxParams p) {
+  constexpr int kPer = kVcMaxTokens / 32;  // scores per lane
+  grid_dependency_wait();  // the partial scores come from the projection
+  grid_launch_dependents();
+  const int f = blockIdx.x, c = blockIdx.y * kVcSoftmaxWarps + (threadIdx.x >> 5);
+  const int lane = threadIdx.x & 31;
+  if (c >= p.C) return;
+  const long long row = static_cast<long long>(c) * p.F * p.N + static_cast<long long>(f) * p.N;
+  float x[kPer];
+#pragma unroll
+  for (int i = 0; i < kPer; ++i) {
+    const int n = lane + 32 * i;
+    x[i] = n < p.N ? __ldg(p.scores + row + n) : -INFINITY;
+  }
+  // the other hidden-range partials, added in split order
+  for (int s = 1; s < p.ks; ++s) {
+    const float *part = p.scores + s * p.part_stride + row;
+#pragma unroll
+    for (int i = 0; i < kPer; ++i) {
+      const int n = lane + 32 * i;
+      if (n < p.N) x[i] += __ldg(part + n);
+    }
+  }
+  float m = -INFINITY;
+#pragma unroll
+  for (int i = 0; i < kPer; ++i) m = fmaxf(m, x[i]);
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, o));
+  constexpr float kLog2e = 1.4426950408889634f;
+  const float mb = m * kLog2e;
+  __nv_bfloat16 *prow = p.P + static_cast<long long>(c) * p.F * p.Np + static_cast<long long>(f) * p.Np;
+  float l = 0.f;
+#pragma unroll
+  for (int i = 0; i < kPer; ++i) {
+    const int n = lane + 32 * i;
+    if (n < p.Np) {
+      const __nv_bfloat16 b = __float2bfloat16_rn(n < p.N ? fast_exp2(fmaf(x[i], kLog2e, -mb)) : 0.f);
+      l += __bfloat162float(b);
+      prow[n] = b;
+    }
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) l += __shfl_xor_sync(0xffffffffu, l, o);
+  if (lane == 0) p.l[f * p.C + c] = l;
 }
 
 __global__ void __launch_bounds__(kVcThreads, 1)
-compress_apply_kernel(const __grid_constant__ CUtensorMap tmap_f, const __grid_constant__ VcParams p) {
+compress_apply_kernel(const __grid_constant__ CUtensorMap tmap_f, const __grid_constant__ CUtensorMap tmap_p,
+                      const __grid_constant__ VcParams p) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t *smem = reinterpret_cast<uint8_t *>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
-  const uint32_t fv = smem_addr(smem);
-  const uint32_t half_bytes = static_cast<uint32_t>(p.Npad) * 128u;
-  uint64_t *bar_mem = reinterpret_cast<uint64_t *>(smem + 2 * static_cast<size_t>(half_bytes));
-  int *s_misc = reinterpret_cast<int *>(bar_mem + 3);  // [0] TMEM base, [1] abort, [2] copies issued
+  const int S = p.stages;
+  const uint32_t ring = smem_addr(smem);
+  uint64_t *bar_mem = reinterpret_cast<uint64_t *>(smem + static_cast<size_t>(S) * p.stage_bytes);
+  int *s_misc = reinterpret_cast<int *>(bar_mem + 2 * S + 1);  // [0] TMEM, [1] abort, [2] issued, [3] consumed
+  float *s_inv = reinterpret_cast<float *>(s_misc + 16);       // 1 / l of the frame's queries
   volatile int *s_abort = s_misc + 1;
-  const uint32_t FVFULL = smem_addr(bar_mem), PFULL = FVFULL + 8, ODONE = FVFULL + 16;
+  const uint32_t bars = smem_addr(bar_mem);
+  const int FULL = 0, EMPTY = S, DONE = 2 * S;
+  auto bar = [&](int i) -> uint32_t { return bars + 8u * static_cast<uint32_t>(i); };
 
   const int chunk = blockIdx.x, f = blockIdx.y;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
 
   grid_launch_dependents();
   if (tid == 0) {
-    mbar_init(FVFULL, 1);
-    mbar_init(PFULL, 128);
-    mbar_init(ODONE, 1);
+    for (int i = 0; i < S; ++i) {
+      mbar_init(bar(FULL + i), 1);
+      mbar_init(bar(EMPTY + i), 1);
+    }
+    mbar_init(bar(DONE), 1);
     fence_mbar_init();
     prefetch_tensormap(&tmap_f);
+    prefetch_tensormap(&tmap_p);
     s_misc[1] = 0;
     s_misc[2] = 0;
+    s_misc[3] = 0;
   }
   if (warp == kVcMmaWarp) {
-    tmem_alloc(smem_addr(s_misc), kVcTmemCols);
+    tmem_alloc(smem_addr(s_misc), p.tmem_cols);
     tmem_relinquish_alloc_permit();
     tc_fence_before_sync();
   }
@@ -95,106 +167,79 @@ compress_apply_kernel(const __grid_constant__ CUtensorMap tmap_f, const __grid_c
 
   if (warp == kVcProducerWarp) {
     if (lane == 0) {
-      // the features may come from the previous kernel on the stream
-      grid_dependency_wait();
+      grid_dependency_wait();  // P comes from the softmax kernel
       const uint64_t pol = l2_policy_evict_first();
-      mbar_arrive_expect_tx(FVFULL, 2 * half_bytes);
-      for (int h = 0; h < 2; ++h)
-        for (int t0 = 0; t0 < p.Npad; t0 += p.BT)
-          tma_load_2d(fv + h * half_bytes + static_cast<uint32_t>(t0) * 128u, &tmap_f,
-                      chunk * kVcCols + h * 64, f * p.N + t0, FVFULL, pol);
-      s_misc[2] = 1;
+      int k = 0;
+      for (; k < p.KT; ++k) {
+        const int slot = k % S;
+        if (k >= S && !mbar_wait_or_abort(bar(EMPTY + slot), ((k / S) - 1) & 1, s_abort)) break;
+        const uint32_t dst = ring + static_cast<uint32_t>(slot) * p.stage_bytes;
+        mbar_arrive_expect_tx(bar(FULL + slot), p.stage_bytes);
+        // features: tokens f*N + 64k .. +63 of columns [128 chunk, +64) and [+64, +128)
+        tma_load_2d(dst, &tmap_f, chunk * kVcCols, f * p.N + k * kVcTokens, bar(FULL + slot), pol);
+        tma_load_2d(dst + kVcFBytes / 2, &tmap_f, chunk * kVcCols + 64, f * p.N + k * kVcTokens,
+                    bar(FULL + slot), pol);
+        // weights of those tokens for every query (rows >= C are zero-filled)
+        tma_load_2d(dst + kVcFBytes, &tmap_p, f * p.Np + k * kVcTokens, 0, bar(FULL + slot), pol);
+      }
+      s_misc[2] = k;
     }
     __syncwarp();
   } else if (warp == kVcMmaWarp) {
-    int w = 1;
-    if (lane == 0)
-      w = mbar_wait_or_abort(PFULL, 0, s_abort) && mbar_wait_or_abort(FVFULL, 0, s_abort);
-    if (__shfl_sync(0xffffffffu, w, 0)) {
+    const uint32_t idesc = idesc_bf16_f32(128, p.Cp, 1, 0);  // A MN-major, B K-major
+    bool ok = true;
+    for (int k = 0; k < p.KT; ++k) {
+      const int slot = k % S;
+      int w = 1;
+      if (lane == 0) w = mbar_wait_or_abort(bar(FULL + slot), (k / S) & 1, s_abort);
+      if (!__shfl_sync(0xffffffffu, w, 0)) {
+        ok = false;
+        break;
+      }
       tc_fence_after_sync();
-      constexpr uint32_t kIdesc = idesc_bf16_f32(128, kVcCols, 0, 1);  // P from TMEM, F_V MN-major
+      if (lane == 0) s_misc[3] = k + 1;
+      const uint32_t base = ring + static_cast<uint32_t>(slot) * p.stage_bytes;
       if (elect_one()) {
-        for (int s = 0; s < p.Npad / 16; ++s) {
-          // 16 tokens = two 8-row swizzle atoms (2 KB) per half; the two
-          // 64-column halves of N are half_bytes apart
-          const uint64_t b = smem_desc_sw128(fv + static_cast<uint32_t>(s) * 2048u, half_bytes, 1024);
-          tc_mma_ts(tmem + kVcTmemO, tmem + kVcTmemP + static_cast<uint32_t>(s) * 8u, b, kIdesc,
-                    s > 0 ? 1u : 0u);
+#pragma unroll
+        for (int kk = 0; kk < kVcTokens / 16; ++kk) {
+          // A: 16 tokens = two 8-row atoms (2 KB) into each 64-column half;
+          // the halves (M) are kVcFBytes / 2 apart.  B: 16 tokens = 32 bytes
+          // along the 128-byte swizzled rows of P, 8-row groups 1 KB apart.
+          const uint64_t a = smem_desc_sw128(base + kk * 2048u, kVcFBytes / 2, 1024);
+          const uint64_t b = smem_desc_sw128(base + kVcFBytes + kk * 32u, 16, 1024);
+          tc_mma_ss(tmem, a, b, idesc, (k > 0 || kk > 0) ? 1u : 0u);
         }
-        tc_commit(ODONE);
+        tc_commit(bar(EMPTY + slot));
       }
       __syncwarp();
-      // every MMA has completed before the teardown frees TMEM
-      (void)mbar_wait_bounded(ODONE, 0);
     }
+    if (ok && elect_one()) tc_commit(bar(DONE));
+    __syncwarp();
+    if (ok) (void)mbar_wait_bounded(bar(DONE), 0);
   } else {
     // ------------------------------------------------------------------
-    // weights and output: thread = query c = TMEM lane
+    // epilogue: lane = feature column 32 * warp + lane of the chunk, TMEM
+    // columns = queries
     // ------------------------------------------------------------------
-    const int c = 32 * warp + lane;
-    const bool valid = c < p.C;
-    const bool warp_used = 32 * warp < p.C;
-    const uint32_t lane_base = tmem + (static_cast<uint32_t>(32 * warp) << 16);
-    grid_dependency_wait();  // the scores come from the previous kernel
-    float l = 0.f;
-    if (warp_used) {
-      const float *srow = p.scores + (valid ? c : 0) * p.score_stride + static_cast<long long>(f) * p.N;
-      float m = -INFINITY;
-      if (valid) {
-        if (p.vec4) {
-          for (int n = 0; n < p.N; n += 4) {
-            const float4 v = __ldg(reinterpret_cast<const float4 *>(srow + n));
-            m = fmaxf(m, fmaxf(fmaxf(v.x, v.y), fmaxf(v.z, v.w)));
-          }
-        } else {
-          for (int n = 0; n < p.N; ++n) m = fmaxf(m, __ldg(srow + n));
-        }
-      }
-      constexpr float kLog2e = 1.4426950408889634f;
-      const float mb = m * kLog2e;
-      // 64 tokens (32 TMEM columns of bf16 pairs) per store
-      for (int g = 0; g < (p.Npad + 63) / 64; ++g) {
-        uint32_t pk[32];
-#pragma unroll
-        for (int j = 0; j < 32; ++j) {
-          const int n0 = g * 64 + 2 * j;
-          float e0 = 0.f, e1 = 0.f;
-          if (valid && n0 < p.N) e0 = fast_exp2(fmaf(__ldg(srow + n0), kLog2e, -mb));
-          if (valid && n0 + 1 < p.N) e1 = fast_exp2(fmaf(__ldg(srow + n0 + 1), kLog2e, -mb));
-          const __nv_bfloat16 b0 = __float2bfloat16_rn(e0), b1 = __float2bfloat16_rn(e1);
-          l += __bfloat162float(b0) + __bfloat162float(b1);
-          pk[j] = static_cast<uint32_t>(__bfloat16_as_ushort(b0)) |
-                  (static_cast<uint32_t>(__bfloat16_as_ushort(b1)) << 16);
-        }
-        tmem_st_32x32b_x32(lane_base + kVcTmemP + static_cast<uint32_t>(g) * 32u, pk);
-      }
-      tmem_wait_st();
+    grid_dependency_wait();  // l comes from the softmax kernel
+    for (int c = tid; c < p.C; c += 128) {
+      const float l = p.l[f * p.C + c];
+      s_inv[c] = l > 0.f ? 1.f / l : 0.f;
     }
-    tc_fence_before_sync();
-    mbar_arrive(PFULL);
-
-    bool ok = mbar_wait_or_abort(ODONE, 0, s_abort);
+    named_bar_sync(1, 128);
+    bool ok = mbar_wait_or_abort(bar(DONE), 0, s_abort);
     ok = __all_sync(0xffffffffu, ok);
-    if (ok && warp_used) {
+    if (ok) {
       tc_fence_after_sync();
-      const float inv = valid && l > 0.f ? 1.f / l : 0.f;
-#pragma unroll 1
-      for (int h = 0; h < 2; ++h) {
-        uint32_t v[64];
-        tmem_ld_32x32b_x64(lane_base + kVcTmemO + static_cast<uint32_t>(h) * 64u, v);
-        if (valid) {
-          uint4 *dst = reinterpret_cast<uint4 *>(
-              p.out + (static_cast<size_t>(f) * p.C + c) * p.d + chunk * kVcCols + h * 64);
+      const uint32_t lane_base = tmem + (static_cast<uint32_t>(32 * warp) << 16);
+      __nv_bfloat16 *dst = p.out + static_cast<size_t>(f) * p.C * p.d + chunk * kVcCols + 32 * warp + lane;
+      for (int c0 = 0; c0 < p.Cp; c0 += 16) {
+        uint32_t v[16];
+        tmem_ld_32x32b_x16(lane_base + static_cast<uint32_t>(c0), v);
 #pragma unroll
-          for (int q = 0; q < 8; ++q) {
-            uint4 w4;
-            w4.x = pack_bf16x2(__uint_as_float(v[8 * q + 0]) * inv, __uint_as_float(v[8 * q + 1]) * inv);
-            w4.y = pack_bf16x2(__uint_as_float(v[8 * q + 2]) * inv, __uint_as_float(v[8 * q + 3]) * inv);
-            w4.z = pack_bf16x2(__uint_as_float(v[8 * q + 4]) * inv, __uint_as_float(v[8 * q + 5]) * inv);
-            w4.w = pack_bf16x2(__uint_as_float(v[8 * q + 6]) * inv, __uint_as_float(v[8 * q + 7]) * inv);
-            dst[q] = w4;
-          }
-        }
+        for (int j = 0; j < 16; ++j)
+          if (c0 + j < p.C)
+            dst[static_cast<size_t>(c0 + j) * p.d] = __float2bfloat16_rn(__uint_as_float(v[j]) * s_inv[c0 + j]);
       }
     }
     tc_fence_before_sync();
@@ -204,13 +249,13 @@ compress_apply_kernel(const __grid_constant__ CUtensorMap tmap_f, const __grid_c
   __syncthreads();
   if (*s_abort) {
     if (tid == 0) set_status(p.status, SF_DEVICE_TIMEOUT);
-    // copies issued but never consumed: wait (bounded) until they land
-    if (warp == kVcProducerWarp && lane == 0 && s_misc[2]) (void)mbar_wait_bounded(FVFULL, 0);
+    if (warp == kVcProducerWarp && lane == 0)
+      for (int k = s_misc[3]; k < s_misc[2]; ++k) (void)mbar_wait_bounded(bar(FULL + k % S), (k / S) & 1);
     __syncthreads();
   }
   if (warp == kVcMmaWarp) {
     tc_fence_after_sync();
-    tmem_dealloc(tmem, kVcTmemCols);
+    tmem_dealloc(tmem, p.tmem_cols);
   }
 }
 
@@ -224,23 +269,30 @@ static int vc_setup(const DeviceInfo &dev) {
   std::lock_guard<std::mutex> lock(mu);
   if (done[dev.ordinal]) return SF_OK;
   cudaError_t e = cudaFuncSetAttribute(compress_apply_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       static_cast<int>(vc_smem_bytes(kVcMaxTokens)));
+                                       dev.max_smem_optin);
   if (e != cudaSuccess) return fail(SF_ERR_CUDA, "cudaFuncSetAttribute (compressor): %s", cudaGetErrorString(e));
   done[dev.ordinal] = true;
   return SF_OK;
 }
 
-// Token rows per TMA box: the largest multiple of 16 that divides Npad and
-// is at most 256 (boxes tile each half exactly, 1024-byte aligned).
-static int box_tokens(int Npad) {
-  const int k = Npad / 16;
-  int q = 16;
-  while (k % q) --q;
-  return 16 * q;
-}
+struct VcLayout {
+  int ks;
+  size_t scores, P, l, total;
+};
 
-static size_t vc_workspace(int F, int N, int C) {
-  return 256 + round_up(static_cast<size_t>(C) * F * N * sizeof(float), 256);
+static VcLayout vc_layout(int F, int N, int C, int d, int sm_count) {
+  VcLayout L;
+  L.ks = projection_splits(F * N, d, sm_count);
+  const int Np = (N + kVcTokens - 1) / kVcTokens * kVcTokens;
+  size_t off = 256;
+  L.scores = off;
+  off = round_up(off + static_cast<size_t>(L.ks) * C * F * N * sizeof(float), 256);
+  L.P = off;
+  off = round_up(off + static_cast<size_t>(C) * F * Np * 2, 256);
+  L.l = off;
+  off = round_up(off + static_cast<size_t>(F) * C * sizeof(float), 256);
+  L.total = off;
+  return L;
 }
 
 static int check_vc(const void *queries, const void *features, int F, int N, int C, int d, const void *out) {
@@ -261,9 +313,12 @@ static int check_vc(const void *queries, const void *features, int F, int N, int
 
 extern "C" {
 
-size_t sf_visual_compress_workspace_size(int F, int N, int C) {
-  if (F < 1 || N < 1 || C < 1 || N > sf::kVcMaxTokens || C > sf::kVcMaxQueries) return 0;
-  return sf::vc_workspace(F, N, C);
+size_t sf_visual_compress_workspace_size(int F, int N, int C, int d) {
+  using namespace sf;
+  if (F < 1 || N < 1 || C < 1 || N > kVcMaxTokens || C > kVcMaxQueries || d < kVcCols) return 0;
+  DeviceInfo dev;
+  if (current_device(&dev) != SF_OK) return 0;
+  return vc_layout(F, N, C, d, dev.sm_count).total;
 }
 
 int sf_visual_compress(const void *queries, const void *features, int F, int N, int C, int d,
@@ -272,55 +327,94 @@ int sf_visual_compress(const void *queries, const void *features, int F, int N, 
   clear_error();
   int st = check_vc(queries, features, F, N, C, d, out);
   if (st != SF_OK) return st;
-  if (!workspace || !aligned(workspace, 256))
-    return fail(SF_ERR_WORKSPACE, "workspace must be non-NULL and 256-byte aligned");
-  const size_t need = vc_workspace(F, N, C);
-  if (workspace_bytes < need)
-    return fail(SF_ERR_WORKSPACE, "workspace has %zu bytes, needs %zu", workspace_bytes, need);
   DeviceInfo dev;
   st = current_device(&dev);
   if (st != SF_OK) return st;
   if (dev.cc_major != 10) return fail(SF_ERR_UNSUPPORTED, "the compressor needs an sm_10x GPU");
+  if (!workspace || !aligned(workspace, 256))
+    return fail(SF_ERR_WORKSPACE, "workspace must be non-NULL and 256-byte aligned");
+  const VcLayout L = vc_layout(F, N, C, d, dev.sm_count);
+  if (workspace_bytes < L.total)
+    return fail(SF_ERR_WORKSPACE, "workspace has %zu bytes, needs %zu", workspace_bytes, L.total);
   st = vc_setup(dev);
   if (st != SF_OK) return st;
 
   uint8_t *ws = static_cast<uint8_t *>(workspace);
   uint32_t *status = reinterpret_cast<uint32_t *>(ws);
-  float *scores = reinterpret_cast<float *>(ws + 256);
-  // 1. S = Q F_V^T over all frames: [C][F*N]
-  st = launch_projection(queries, features, C, d, F * N, scores, status, true, true, stream);
+  float *scores = reinterpret_cast<float *>(ws + L.scores);
+  __nv_bfloat16 *P = reinterpret_cast<__nv_bfloat16 *>(ws + L.P);
+  float *lsum = reinterpret_cast<float *>(ws + L.l);
+  const int Np = (N + kVcTokens - 1) / kVcTokens * kVcTokens;
+
+  // 1. partial scores S_s = Q F_V^T over hidden range s, all frames: [ks][C][F*N]
+  st = launch_projection(queries, features, C, d, F * N, scores, status, true, true, L.ks, stream);
   if (st != SF_OK) return st;
 
-  // 2. per (128 columns, frame): softmax over the frame's tokens and P F_V
-  VcParams prm;
-  prm.scores = scores;
-  prm.out = static_cast<__nv_bfloat16 *>(out);
-  prm.status = status;
-  prm.score_stride = static_cast<long long>(F) * N;
-  prm.F = F;
-  prm.N = N;
-  prm.C = C;
-  prm.d = d;
-  prm.Npad = (N + 15) / 16 * 16;
-  prm.BT = box_tokens(prm.Npad);
-  prm.vec4 = N % 4 == 0 ? 1 : 0;
-  CUtensorMap tmap;
-  const uint64_t dims[2] = {static_cast<uint64_t>(d), static_cast<uint64_t>(F) * N};
-  const uint64_t strides[1] = {static_cast<uint64_t>(d) * 2};
-  const uint32_t box[2] = {64, static_cast<uint32_t>(prm.BT)};
-  st = encode_tensor_map_bf16(&tmap, features, 2, dims, strides, box);
-  if (st != SF_OK) return st;
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(d / kVcCols, F);
-  cfg.blockDim = dim3(kVcThreads);
-  cfg.dynamicSmemBytes = vc_smem_bytes(prm.Npad);
   cfg.stream = stream;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  cudaError_t e = cudaLaunchKernelEx(&cfg, compress_apply_kernel, tmap, prm);
+
+  // 2. weights P = bf16(exp(S - max)) and their sums l
+  VcSoftmaxParams sp;
+  sp.scores = scores;
+  sp.P = P;
+  sp.l = lsum;
+  sp.part_stride = static_cast<long long>(C) * F * N;
+  sp.ks = L.ks;
+  sp.F = F;
+  sp.N = N;
+  sp.C = C;
+  sp.Np = Np;
+  cfg.gridDim = dim3(F, (C + kVcSoftmaxWarps - 1) / kVcSoftmaxWarps);
+  cfg.blockDim = dim3(32 * kVcSoftmaxWarps);
+  cfg.dynamicSmemBytes = 0;
+  cudaError_t e = cudaLaunchKernelEx(&cfg, compress_softmax_kernel, sp);
+  if (e != cudaSuccess) return fail(SF_ERR_CUDA, "compressor softmax launch: %s", cudaGetErrorString(e));
+
+  // 3. O^T = F_V^T P^T per (128 columns, frame), divided by l
+  VcParams prm;
+  prm.l = lsum;
+  prm.out = static_cast<__nv_bfloat16 *>(out);
+  prm.status = status;
+  prm.F = F;
+  prm.N = N;
+  prm.C = C;
+  prm.Cp = (C + 15) / 16 * 16;
+  prm.d = d;
+  prm.Np = Np;
+  prm.KT = Np / kVcTokens;
+  prm.stage_bytes = kVcFBytes + static_cast<uint32_t>(prm.Cp) * 128u;
+  // a ring no deeper than the CTA's token chunks, and small enough for two
+  // or more CTAs per SM (the CTAs are short: prologue and epilogue overlap)
+  prm.stages = prm.KT < kVcMaxStages ? prm.KT : kVcMaxStages;
+  while (prm.stages > 2 && vc_smem_bytes(prm.stages, prm.stage_bytes, C) > static_cast<size_t>(dev.max_smem_optin) / 2)
+    --prm.stages;
+  uint32_t cols = 32;
+  while (cols < static_cast<uint32_t>(prm.Cp)) cols <<= 1;
+  prm.tmem_cols = cols;
+  CUtensorMap tmap_f, tmap_p;
+  {
+    const uint64_t dims[2] = {static_cast<uint64_t>(d), static_cast<uint64_t>(F) * N};
+    const uint64_t strides[1] = {static_cast<uint64_t>(d) * 2};
+    const uint32_t box[2] = {64, static_cast<uint32_t>(kVcTokens)};
+    st = encode_tensor_map_bf16(&tmap_f, features, 2, dims, strides, box);
+    if (st != SF_OK) return st;
+  }
+  {
+    const uint64_t dims[2] = {static_cast<uint64_t>(F) * Np, static_cast<uint64_t>(C)};
+    const uint64_t strides[1] = {static_cast<uint64_t>(F) * Np * 2};
+    const uint32_t box[2] = {static_cast<uint32_t>(kVcTokens), static_cast<uint32_t>(prm.Cp)};
+    st = encode_tensor_map_bf16(&tmap_p, P, 2, dims, strides, box);
+    if (st != SF_OK) return st;
+  }
+  cfg.gridDim = dim3(d / kVcCols, F);
+  cfg.blockDim = dim3(kVcThreads);
+  cfg.dynamicSmemBytes = vc_smem_bytes(prm.stages, prm.stage_bytes, C);
+  e = cudaLaunchKernelEx(&cfg, compress_apply_kernel, tmap_f, tmap_p, prm);
   if (e != cudaSuccess) return fail(SF_ERR_CUDA, "compressor launch: %s", cudaGetErrorString(e));
   return SF_OK;
 }

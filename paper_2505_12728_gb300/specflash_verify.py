@@ -97,7 +97,7 @@ def load_library(path: str | None = None):
         lib.sf_sample.restype = I
         lib.sf_draft_sample.argtypes = [P, P, P, P, I, I, I, P, P, P, P, S, P]
         lib.sf_draft_sample.restype = I
-        lib.sf_visual_compress_workspace_size.argtypes = [I, I, I]
+        lib.sf_visual_compress_workspace_size.argtypes = [I, I, I, I]
         lib.sf_visual_compress_workspace_size.restype = S
         lib.sf_visual_compress.argtypes = [P, P, I, I, I, I, P, P, S, P]
         lib.sf_visual_compress.restype = I
@@ -379,8 +379,8 @@ def draft_sample(hidden, weight, uniforms, temperature, *, logits=None, probs=No
 # --------------------------------------------------------------------------- #
 # visual token compression                                                    #
 # --------------------------------------------------------------------------- #
-def visual_compress_workspace_size(F, N, C) -> int:
-    n = load_library().sf_visual_compress_workspace_size(F, N, C)
+def visual_compress_workspace_size(F, N, C, d) -> int:
+    n = load_library().sf_visual_compress_workspace_size(F, N, C, d)
     if n == 0:
         raise SFError(1, "invalid compressor shape")
     return int(n)
@@ -399,7 +399,7 @@ def visual_compress(queries, features, *, out=None, workspace=None, stream=None)
         out = torch.empty((F, C, d), dtype=torch.bfloat16, device=queries.device)
     _need(out, "out", torch.bfloat16, (F, C, d))
     if workspace is None:
-        workspace = new_workspace(visual_compress_workspace_size(F, N, C), queries.device)
+        workspace = new_workspace(visual_compress_workspace_size(F, N, C, d), queries.device)
     _check(load_library().sf_visual_compress(_ptr(queries), _ptr(features), F, N, C, d, _ptr(out),
                                              _ptr(workspace), workspace.numel(),
                                              _stream_handle(stream)))

@@ -25,7 +25,7 @@ def _gpu():
 
 
 def run(queries, features):
-    ws = sfv.new_workspace(sfv.visual_compress_workspace_size(*features.shape[:2], queries.shape[0]))
+    ws = sfv.new_workspace(sfv.visual_compress_workspace_size(*features.shape[:2], *queries.shape))
     out = sfv.visual_compress(bf16_tensor(queries), bf16_tensor(features), workspace=ws)
     torch.cuda.synchronize()
     assert sfv.read_device_status(ws) == 0
@@ -122,7 +122,7 @@ def test_compressor_invalid_arguments():
     q = torch.zeros((4, 128), dtype=torch.bfloat16, device="cuda")
     f = torch.zeros((1, 8, 128), dtype=torch.bfloat16, device="cuda")
     out = torch.zeros((1, 4, 128), dtype=torch.bfloat16, device="cuda")
-    ws = sfv.new_workspace(sfv.visual_compress_workspace_size(1, 8, 4))
+    ws = sfv.new_workspace(sfv.visual_compress_workspace_size(1, 8, 4, 128))
     P = lambda t: t.data_ptr()
     n = ws.numel()
     assert lib.sf_visual_compress(P(q), P(f), 1, 8, 4, 128, P(out), P(ws), n, None) == 0
@@ -131,5 +131,5 @@ def test_compressor_invalid_arguments():
     assert lib.sf_visual_compress(P(q), P(f), 1, 8, 4, 96, P(out), P(ws), n, None) == 1
     assert lib.sf_visual_compress(P(q), P(f), 0, 8, 4, 128, P(out), P(ws), n, None) == 1
     assert lib.sf_visual_compress(P(q), P(f), 1, 8, 4, 128, P(out), P(ws), 16, None) == 4
-    assert lib.sf_visual_compress_workspace_size(1, 769, 4) == 0
+    assert lib.sf_visual_compress_workspace_size(1, 769, 4, 128) == 0
     torch.cuda.synchronize()
