@@ -202,6 +202,33 @@ int sf_accept(const float *target_logits, const float *draft_probs,
               cudaStream_t stream);
 
 /* ------------------------------------------------------------------------ */
+/* Fused target LM head + acceptance (Sec. 3.1: the target scores the K     */
+/* candidates in one forward pass; its LM head turns the k+1 verified       */
+/* positions' final hidden states into the logits the rule above reads).   */
+/* target_logits[b][i][v] = sum_j hidden[b][i][j] * weight[v][j] (bf16 in,  */
+/* fp32 accumulate), then exactly the rule of sf_accept, with the rows'     */
+/* max, argmax and softmax sums reduced in the projection's epilogue        */
+/* instead of a second pass over the logits.                                */
+/*                                                                           */
+/* hidden        bf16 [B][k+1][d], 16-byte aligned.                          */
+/* weight        bf16 [V][d] (the target's LM head), 16-byte aligned.        */
+/* logits        fp32 [B][k+1][V], output (also read by the draw).           */
+/* other arguments and outputs as for sf_accept.                             */
+/* Limits: those of sf_accept, B * (k + 1) <= 256, d a multiple of 8 in    */
+/* [8, 2^20].  workspace >= sf_verify_lm_head_accept_workspace_size(B, k, V)*/
+/* bytes, 256-byte aligned, zero-filled before first use.                   */
+/* The weight copies start before the previous kernel on the stream        */
+/* completes (the weights must not be written by it).                       */
+/* ------------------------------------------------------------------------ */
+size_t sf_verify_lm_head_accept_workspace_size(int B, int k, int V);
+
+int sf_verify_lm_head_accept(const void *hidden, const void *weight, const float *draft_probs,
+                             const int32_t *draft_tokens, const float *uniforms,
+                             const float *temperature, int B, int k, int V, int d, float *logits,
+                             int32_t *num_accepted, int32_t *out_tokens, float *accept_ratio,
+                             void *workspace, size_t workspace_bytes, cudaStream_t stream);
+
+/* ------------------------------------------------------------------------ */
 /* KV commit after acceptance (Sec. 3.1: the accepted candidates join the    */
 /* context and decoding continues from the first rejected position; Sec.    */
 /* 3.3: the next draft block starts from the emitted token).  The paper      */

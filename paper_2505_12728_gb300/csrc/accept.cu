@@ -112,6 +112,56 @@ __device__ __forceinline__ void draw_terms(float x, float qx, bool residual, flo
   r = residual ? fmaxf(__fsub_rn(pz, qx), 0.0f) : pz;
 }
 
+// The k accept/reject decisions of sequence b and its outputs, from the
+// combined rows in shared memory (row rr: max s_rm, first argmax s_rarg,
+// float-float sum s_rS, the draft token's logit s_rlx and draft probability
+// s_rqx, s_rhx = the token lies in [0, V)).  Called by every thread of the
+// block after the rows are visible; thread i < k tests draft i (my_tok,
+// my_u), threads <= k write out_tokens; j goes to num_accepted and seqs.
+__device__ void decide_sequence(const AccParams &p, int b, bool greedy, float tau, int my_tok,
+                                float my_u, const float *s_rm, const int *s_rarg, const ff *s_rS,
+                                const float *s_rlx, const float *s_rqx, const int *s_rhx,
+                                int *s_acc) {
+  const int tid = threadIdx.x, k = p.k, V = p.V;
+  if (tid < k) {
+    const int i = tid, x = my_tok;
+    int acc = 0;
+    float ratio = 0.f;
+    if (x < 0 || x >= V || !s_rhx[i]) {
+      set_status(p.status, SF_DEVICE_BAD_TOKEN);  // treated as a rejection
+    } else if (greedy) {
+      acc = (x == s_rarg[i]);
+      ratio = acc ? 1.f : 0.f;
+    } else {
+      // p(x) = exp((l_x - m) / tau) / S; accept iff u * q(x) < p(x), with the
+      // product u * q kept exactly as float-float
+      const float px = ff_div_to_f(exp_diff_accurate(s_rlx[i], s_rm[i], tau), s_rS[i]);
+      const float qd = s_rqx[i];
+      const float uq = __fmul_rn(my_u, qd);
+      const ff uqf = ff{uq, __fmaf_rn(my_u, qd, -uq)};
+      acc = ff_lt(uqf, ff_of(px)) ? 1 : 0;
+      ratio = qd > 0.f ? fminf(1.f, __fdiv_rn(px, qd)) : 1.f;
+    }
+    s_acc[i] = acc;
+    if (p.ratio) p.ratio[(size_t)b * k + i] = ratio;
+  }
+  __syncthreads();
+  if (tid <= k) {
+    // every writer finds j in shared memory; thread i writes out_tokens[i]
+    int j = k;
+    for (int i = 0; i < k; ++i)
+      if (!s_acc[i]) { j = i; break; }
+    int32_t v = -1;
+    if (tid < j) v = my_tok;
+    else if (tid == j && greedy) v = s_rarg[j];
+    if (!(tid == j && !greedy)) p.out_tokens[(size_t)b * (k + 1) + tid] = v;
+    if (tid == 0) {
+      p.num_accepted[b] = j;
+      p.seqs[b].j = j;
+    }
+  }
+}
+
 __global__ void __launch_bounds__(kAccThreads)
 accept_stats_kernel(const __grid_constant__ AccParams p) {
   __shared__ ff s_d[32];
@@ -249,44 +299,59 @@ accept_stats_kernel(const __grid_constant__ AccParams p) {
     }
   }
   __syncthreads();
+  decide_sequence(p, b, greedy, tau, my_tok, my_u, s_rm, s_rarg, s_rS, s_rlx, s_rqx, s_rhx, s_acc);
+  if (tid == 0) p.seq_tickets[b] = 0u;
+}
+
+// Fused path: the decisions from the projection's per-CTA row statistics
+// (launch_projection_stats, G records per row) instead of a pass over the
+// logits.  grid (B), kAccThreads threads: warp w combines rows w, w + 8, ...
+__global__ void __launch_bounds__(kAccThreads)
+accept_decide_kernel(const __grid_constant__ AccParams p, const SampStat *__restrict__ stats, int G) {
+  __shared__ int s_acc[SF_MAX_DRAFT];
+  __shared__ float s_rm[SF_MAX_DRAFT + 1], s_rlx[SF_MAX_DRAFT + 1], s_rqx[SF_MAX_DRAFT + 1];
+  __shared__ int s_rarg[SF_MAX_DRAFT + 1], s_rhx[SF_MAX_DRAFT + 1];
+  __shared__ ff s_rS[SF_MAX_DRAFT + 1];
+  grid_dependency_wait();  // statistics and logits come from the projection
+  grid_launch_dependents();
+  const int b = blockIdx.x, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int k = p.k, V = p.V;
+  const float tau = p.tau[b];
+  const bool greedy = !(tau > 0.0f);
+  int my_tok = -1;
+  float my_u = 0.f;
   if (tid < k) {
-    const int i = tid, x = my_tok;
-    int acc = 0;
-    float ratio = 0.f;
-    if (x < 0 || x >= V || !s_rhx[i]) {
-      set_status(p.status, SF_DEVICE_BAD_TOKEN);  // treated as a rejection
-    } else if (greedy) {
-      acc = (x == s_rarg[i]);
-      ratio = acc ? 1.f : 0.f;
-    } else {
-      // p(x) = exp((l_x - m) / tau) / S; accept iff u * q(x) < p(x), with the
-      // product u * q kept exactly as float-float
-      const float px = ff_div_to_f(exp_diff_accurate(s_rlx[i], s_rm[i], tau), s_rS[i]);
-      const float qd = s_rqx[i];
-      const float uq = __fmul_rn(my_u, qd);
-      const ff uqf = ff{uq, __fmaf_rn(my_u, qd, -uq)};
-      acc = ff_lt(uqf, ff_of(px)) ? 1 : 0;
-      ratio = qd > 0.f ? fminf(1.f, __fdiv_rn(px, qd)) : 1.f;
+    my_tok = p.tokens[(size_t)b * k + tid];
+    my_u = p.u[(size_t)b * (k + 1) + tid];
+  }
+  for (int rr = warp; rr <= k; rr += kAccWarps) {
+    const size_t row = (size_t)b * (k + 1) + rr;
+    const SampStat *cr = stats + row * G;
+    float mv = -INFINITY;
+    int mi = INT_MAX;
+    for (int c = lane; c < G; c += 32)
+      if (better(cr[c].m, cr[c].arg, mv, mi)) { mv = cr[c].m; mi = cr[c].arg; }
+    warp_argmax(mv, mi);
+    ff Sr = ff_of(0.f);
+    if (!greedy && mv != -INFINITY) {
+      for (int c = lane; c < G; c += 32)
+        if (ff_pos(cr[c].S)) Sr = ff_add(Sr, ff_mul(cr[c].S, exp_diff_accurate(cr[c].m, mv, tau)));
+      Sr = warp_sum_ff(Sr);
     }
-    s_acc[i] = acc;
-    if (p.ratio) p.ratio[(size_t)b * k + i] = ratio;
+    if (lane == 0) {
+      const int x = rr < k ? p.tokens[(size_t)b * k + rr] : -1;
+      const bool ok = x >= 0 && x < V;
+      s_rm[rr] = mv;
+      s_rarg[rr] = mi;
+      s_rS[rr] = Sr;
+      s_rlx[rr] = ok ? p.logits[row * V + x] : 0.f;
+      s_rqx[rr] = ok ? p.q[((size_t)b * k + rr) * V + x] : 0.f;
+      s_rhx[rr] = ok ? 1 : 0;
+      p.rows[row] = RowStat{mv, mi, Sr};
+    }
   }
   __syncthreads();
-  if (tid <= k) {
-    // every writer finds j in shared memory; thread i writes out_tokens[i]
-    int j = k;
-    for (int i = 0; i < k; ++i)
-      if (!s_acc[i]) { j = i; break; }
-    int32_t v = -1;
-    if (tid < j) v = my_tok;
-    else if (tid == j && greedy) v = s_rarg[j];
-    if (!(tid == j && !greedy)) p.out_tokens[(size_t)b * (k + 1) + tid] = v;
-    if (tid == 0) {
-      p.num_accepted[b] = j;
-      p.seqs[b].j = j;
-      p.seq_tickets[b] = 0u;
-    }
-  }
+  decide_sequence(p, b, greedy, tau, my_tok, my_u, s_rm, s_rarg, s_rS, s_rlx, s_rqx, s_rhx, s_acc);
 }
 
 __global__ void __launch_bounds__(kAccThreads)
@@ -596,6 +661,100 @@ int sf_accept(const float *target_logits, const float *draft_probs,
   cfg.numAttrs = 1;
   cudaError_t e = cudaLaunchKernelEx(&cfg, accept_stats_kernel, prm);
   if (e != cudaSuccess) return fail(SF_ERR_CUDA, "accept stats launch: %s", cudaGetErrorString(e));
+  cfg.gridDim = dim3(plan.C2, B);
+  e = cudaLaunchKernelEx(&cfg, accept_draw_kernel, prm);
+  if (e != cudaSuccess) return fail(SF_ERR_CUDA, "accept draw launch: %s", cudaGetErrorString(e));
+  return SF_OK;
+}
+
+size_t sf_verify_lm_head_accept_workspace_size(int B, int k, int V) {
+  using namespace sf;
+  if (check_accept_shapes(B, k, V) != SF_OK || B * (k + 1) > SF_MAX_DRAFT_ROWS) return 0;
+  AccPlan plan;
+  if (plan_accept(B, k, V, &plan) != SF_OK) return 0;
+  DeviceInfo dev;
+  if (current_device(&dev) != SF_OK) return 0;
+  const size_t G = static_cast<size_t>(projection_groups(V, dev.sm_count));
+  return acc_layout(B, k, plan).total + round_up(sizeof(SampStat) * B * (k + 1) * G, 256);
+}
+
+int sf_verify_lm_head_accept(const void *hidden, const void *weight, const float *draft_probs,
+                             const int32_t *draft_tokens, const float *uniforms,
+                             const float *temperature, int B, int k, int V, int d, float *logits,
+                             int32_t *num_accepted, int32_t *out_tokens, float *accept_ratio,
+                             void *workspace, size_t workspace_bytes, cudaStream_t stream) {
+  using namespace sf;
+  clear_error();
+  int st = check_accept_shapes(B, k, V);
+  if (st != SF_OK) return st;
+  if (B * (k + 1) > SF_MAX_DRAFT_ROWS)
+    return fail(SF_ERR_INVALID_ARG, "B*(k+1)=%d above %d rows", B * (k + 1), SF_MAX_DRAFT_ROWS);
+  if (!draft_probs || !draft_tokens || !uniforms || !temperature || !num_accepted || !out_tokens)
+    return fail(SF_ERR_INVALID_ARG, "a required pointer is NULL");
+  if (!aligned(draft_probs, 4) || !aligned(draft_tokens, 4) || !aligned(uniforms, 4) ||
+      !aligned(temperature, 4) || !aligned(num_accepted, 4) || !aligned(out_tokens, 4) ||
+      (accept_ratio && !aligned(accept_ratio, 4)))
+    return fail(SF_ERR_INVALID_ARG, "buffers must be 4-byte aligned");
+  if (!workspace || !aligned(workspace, 256))
+    return fail(SF_ERR_WORKSPACE, "workspace must be non-NULL and 256-byte aligned");
+  AccPlan plan;
+  st = plan_accept(B, k, V, &plan);
+  if (st != SF_OK) return st;
+  DeviceInfo dev;
+  st = current_device(&dev);
+  if (st != SF_OK) return st;
+  const AccLayout lay = acc_layout(B, k, plan);
+  const int R = B * (k + 1);
+  const size_t G = static_cast<size_t>(projection_groups(V, dev.sm_count));
+  const size_t need = lay.total + round_up(sizeof(SampStat) * R * G, 256);
+  if (workspace_bytes < need)
+    return fail(SF_ERR_WORKSPACE, "workspace has %zu bytes, needs %zu", workspace_bytes, need);
+
+  uint8_t *ws = static_cast<uint8_t *>(workspace);
+  SampStat *stats = reinterpret_cast<SampStat *>(ws + lay.total);
+  int Gl = 0;
+  // target logits and their per-CTA row statistics; row b*(k+1)+i uses tau_b
+  st = launch_projection_stats(hidden, weight, R, d, V, logits, temperature, k + 1, stats,
+                               reinterpret_cast<uint32_t *>(ws), &Gl, stream);
+  if (st != SF_OK) return st;
+
+  AccParams prm;
+  prm.logits = logits;
+  prm.q = draft_probs;
+  prm.tokens = draft_tokens;
+  prm.u = uniforms;
+  prm.tau = temperature;
+  prm.num_accepted = num_accepted;
+  prm.out_tokens = out_tokens;
+  prm.ratio = accept_ratio;
+  prm.status = reinterpret_cast<uint32_t *>(ws);
+  prm.seq_tickets = reinterpret_cast<uint32_t *>(ws + lay.seq_tickets);
+  prm.draw_tickets = reinterpret_cast<uint32_t *>(ws + lay.draw_tickets);
+  prm.chunks = reinterpret_cast<ChunkRec *>(ws + lay.chunks);
+  prm.rows = reinterpret_cast<RowStat *>(ws + lay.rows);
+  prm.seqs = reinterpret_cast<SeqState *>(ws + lay.seqs);
+  prm.parts = reinterpret_cast<DrawPart *>(ws + lay.parts);
+  prm.B = B;
+  prm.k = k;
+  prm.V = V;
+  prm.C1 = plan.C1;
+  prm.CV1 = plan.CV1;
+  prm.C2 = plan.C2;
+  prm.CV2 = plan.CV2;
+  prm.vec4 = (V % 4 == 0) && aligned(logits, 16) && aligned(draft_probs, 16);
+
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(B);
+  cfg.blockDim = dim3(kAccThreads);
+  cfg.stream = stream;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  cudaError_t e = cudaLaunchKernelEx(&cfg, accept_decide_kernel, prm,
+                                     static_cast<const SampStat *>(stats), Gl);
+  if (e != cudaSuccess) return fail(SF_ERR_CUDA, "accept decide launch: %s", cudaGetErrorString(e));
   cfg.gridDim = dim3(plan.C2, B);
   e = cudaLaunchKernelEx(&cfg, accept_draw_kernel, prm);
   if (e != cudaSuccess) return fail(SF_ERR_CUDA, "accept draw launch: %s", cudaGetErrorString(e));

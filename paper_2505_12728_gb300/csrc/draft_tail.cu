@@ -69,16 +69,9 @@ constexpr int kSampleUnit = 2048;                      // tokens per statistics 
 constexpr int kSampleSpan = 4096;                      // least tokens per finishing CTA
 constexpr int kMaxStatChunks = 4096;                   // statistics chunks per row
 
-struct SampStat {  // one chunk of one row
-  float m;         // largest logit of the chunk
-  int arg;         // its first index
-  ff S;            // sum of exp((x - m) / tau) over the chunk; 0 for greedy rows
-};
-static_assert(sizeof(SampStat) == 16, "SampStat is 16 bytes");
-
 struct LmParams {
   float *logits;     // [R][V]
-  const float *tau;  // [R]; read only with stats
+  const float *tau;  // temperature of row r: tau[r / tau_div]; read only with stats
   SampStat *stats;   // [R][G], or null for the plain projection
   uint32_t *status;
   int R, V, NP;
@@ -91,6 +84,7 @@ struct LmParams {
   uint32_t idesc;
   int w_after_wait;  // copy the weight rows only after griddepcontrol.wait
   int w_keep;        // weight rows are re-read next: L2 evict_last instead of evict_first
+  int tau_div;       // rows per temperature entry (1: one per row)
   int ks;            // hidden-dimension splits: CTA (g, s) sums chunks [s*KC/ks, (s+1)*KC/ks)
   long long part_stride;  // floats between the ks partial outputs (split s adds s * part_stride)
 };
@@ -301,7 +295,7 @@ lm_head_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
     grid_dependency_wait();  // outputs and temperatures follow the previous kernel
     if (stats) {
       for (int c = tid; c < p.NP; c += kLmEpiThreads) {
-        s_tau[c] = c < p.R ? p.tau[c] : 1.f;
+        s_tau[c] = c < p.R ? p.tau[c / p.tau_div] : 1.f;
         run[c] = SampStat{-INFINITY, INT_MAX, ff_of(0.f)};
       }
     }
@@ -707,7 +701,7 @@ static cudaLaunchConfig_t pdl_config(dim3 grid, dim3 block, size_t smem, cudaStr
 static int launch_lm_head(const void *hidden, const void *weight, int R, int hidden_size, int V,
                           float *logits, const float *temperature, SampStat *stats, uint32_t *status,
                           int *G_out, cudaStream_t stream, bool w_after_wait = false,
-                          bool w_keep = false, int ks = 1) {
+                          bool w_keep = false, int ks = 1, int tau_div = 1) {
   DeviceInfo dev;
   int st = current_device(&dev);
   if (st != SF_OK) return st;
@@ -738,6 +732,7 @@ static int launch_lm_head(const void *hidden, const void *weight, int R, int hid
   prm.w_after_wait = w_after_wait ? 1 : 0;
   prm.w_keep = w_keep ? 1 : 0;
   prm.ks = ks < 1 ? 1 : (ks > prm.KC ? prm.KC : ks);
+  prm.tau_div = tau_div < 1 ? 1 : tau_div;
   prm.part_stride = static_cast<long long>(R) * V;
   if (stats && prm.ks != 1) return fail(SF_ERR_INVALID_ARG, "statistics need an unsplit projection");
   const size_t smem = LmSmem::bytes(prm.stages, prm.stage_bytes, NP);
@@ -781,6 +776,20 @@ static int launch_finish(SampleParams prm, cudaStream_t stream) {
   cudaError_t e = cudaLaunchKernelEx(&cfg, sample_finish_kernel, prm);
   if (e != cudaSuccess) return fail(SF_ERR_CUDA, "sampling launch: %s", cudaGetErrorString(e));
   return SF_OK;
+}
+
+int launch_projection_stats(const void *hidden, const void *weight, int R, int hidden_size, int V,
+                            float *logits, const float *temperature, int rows_per_temperature,
+                            SampStat *stats, uint32_t *status, int *G_out, cudaStream_t stream) {
+  const int st = check_lm_args(hidden, weight, R, hidden_size, V, logits);
+  if (st != SF_OK) return st;
+  return launch_lm_head(hidden, weight, R, hidden_size, V, logits, temperature, stats, status, G_out,
+                        stream, false, false, 1, rows_per_temperature);
+}
+
+int projection_groups(int V, int sm_count) {
+  const int tiles = (V + kLmTileV - 1) / kLmTileV;
+  return tiles < sm_count ? tiles : sm_count;
 }
 
 int projection_splits(int V, int hidden_size, int sm_count) {

@@ -20,6 +20,15 @@ struct ff {       // float-float number hi + lo, |lo| <= ulp(hi) / 2
   float hi, lo;
 };
 
+// Softmax statistics of one chunk of one row: written by the projection
+// epilogue (draft_tail.cu), read by the samplers and the fused acceptance.
+struct SampStat {
+  float m;  // largest logit of the chunk
+  int arg;  // its first index
+  ff S;     // sum of exp((x - m) / tau) over the chunk; 0 for greedy rows
+};
+static_assert(sizeof(SampStat) == 16, "SampStat is 16 bytes");
+
 // (value, index) order for argmax: larger value first, then lower index.
 __device__ __forceinline__ bool better(float v, int i, float bv, int bi) {
   return v > bv || (v == bv && i < bi);

@@ -44,6 +44,17 @@ int launch_projection(const void *rows_r, const void *rows_v, int R, int hidden_
 // Hidden-dimension splits that fill the GPU when V has few 128-row tiles.
 int projection_splits(int V, int hidden_size, int sm_count);
 
+// The projection with softmax statistics in its epilogue: logits [R][V] and,
+// per row and CTA (G = projection_groups(V, SM count) CTAs, CTA g owning
+// rows [g*V/G, (g+1)*V/G)), a 16-byte record {max, first argmax,
+// float-float sum of exp((x - max)/tau)} at stats[r * G + g]; row r uses
+// temperature[r / rows_per_temperature] (<= 0: greedy, no sum).
+struct SampStat;
+int launch_projection_stats(const void *hidden, const void *weight, int R, int hidden_size, int V,
+                            float *logits, const float *temperature, int rows_per_temperature,
+                            SampStat *stats, uint32_t *status, int *G_out, cudaStream_t stream);
+int projection_groups(int V, int sm_count);
+
 inline bool aligned(const void *p, size_t a) {
   return (reinterpret_cast<uintptr_t>(p) % a) == 0;
 }

@@ -33,6 +33,7 @@ EXPORTED_SYMBOLS = (
     "sf_kv_commit_workspace_size", "sf_kv_commit",
     "sf_draft_tail_workspace_size", "sf_lm_head", "sf_sample", "sf_draft_sample",
     "sf_visual_compress_workspace_size", "sf_visual_compress",
+    "sf_verify_lm_head_accept_workspace_size", "sf_verify_lm_head_accept",
 )
 
 _lock = threading.Lock()
@@ -101,6 +102,10 @@ def load_library(path: str | None = None):
         lib.sf_visual_compress_workspace_size.restype = S
         lib.sf_visual_compress.argtypes = [P, P, I, I, I, I, P, P, S, P]
         lib.sf_visual_compress.restype = I
+        lib.sf_verify_lm_head_accept_workspace_size.argtypes = [I, I, I]
+        lib.sf_verify_lm_head_accept_workspace_size.restype = S
+        lib.sf_verify_lm_head_accept.argtypes = [P, P, P, P, P, P, I, I, I, I, P, P, P, P, P, S, P]
+        lib.sf_verify_lm_head_accept.restype = I
         _lib = lib
         return lib
 
@@ -270,6 +275,52 @@ def accept(target_logits, draft_probs, draft_tokens, uniforms, temperature, *,
         _ptr(temperature), B, k, V, _ptr(num_accepted), _ptr(out_tokens), _ptr(accept_ratio),
         _ptr(workspace), workspace.numel(), _stream_handle(stream)))
     return num_accepted, out_tokens, accept_ratio
+
+
+def verify_lm_head_accept_workspace_size(B, k, V) -> int:
+    n = load_library().sf_verify_lm_head_accept_workspace_size(B, k, V)
+    if n == 0:
+        raise SFError(1, "invalid fused acceptance shape")
+    return int(n)
+
+
+def verify_lm_head_accept(hidden, weight, draft_probs, draft_tokens, uniforms, temperature, *,
+                          logits=None, num_accepted=None, out_tokens=None, accept_ratio=None,
+                          workspace=None, stream=None, with_ratio=True):
+    """sf_verify_lm_head_accept: hidden bf16 [B][k+1][d] (the target's final
+    hidden states of the verified positions), weight bf16 [V][d], then the
+    acceptance rule as in accept().  Returns (logits fp32 [B][k+1][V],
+    num_accepted int32 [B], out_tokens int32 [B][k+1], accept_ratio or None)."""
+    B, k1, d = hidden.shape
+    k = k1 - 1
+    V = weight.shape[0]
+    _need(hidden, "hidden", torch.bfloat16)
+    _need(weight, "weight", torch.bfloat16, (V, d))
+    _need(draft_probs, "draft_probs", torch.float32, (B, k, V))
+    _need(draft_tokens, "draft_tokens", torch.int32, (B, k))
+    _need(uniforms, "uniforms", torch.float32, (B, k + 1))
+    _need(temperature, "temperature", torch.float32, (B,))
+    dev = hidden.device
+    if logits is None:
+        logits = torch.empty((B, k + 1, V), dtype=torch.float32, device=dev)
+    if num_accepted is None:
+        num_accepted = torch.empty(B, dtype=torch.int32, device=dev)
+    if out_tokens is None:
+        out_tokens = torch.empty((B, k + 1), dtype=torch.int32, device=dev)
+    if accept_ratio is None and with_ratio:
+        accept_ratio = torch.empty((B, k), dtype=torch.float32, device=dev)
+    _need(logits, "logits", torch.float32, (B, k + 1, V))
+    _need(num_accepted, "num_accepted", torch.int32, (B,))
+    _need(out_tokens, "out_tokens", torch.int32, (B, k + 1))
+    if accept_ratio is not None:
+        _need(accept_ratio, "accept_ratio", torch.float32, (B, k))
+    if workspace is None:
+        workspace = new_workspace(verify_lm_head_accept_workspace_size(B, k, V), dev)
+    _check(load_library().sf_verify_lm_head_accept(
+        _ptr(hidden), _ptr(weight), _ptr(draft_probs), _ptr(draft_tokens), _ptr(uniforms),
+        _ptr(temperature), B, k, V, d, _ptr(logits), _ptr(num_accepted), _ptr(out_tokens),
+        _ptr(accept_ratio), _ptr(workspace), workspace.numel(), _stream_handle(stream)))
+    return logits, num_accepted, out_tokens, accept_ratio
 
 
 def kv_commit_workspace_size() -> int:
