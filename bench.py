@@ -393,6 +393,64 @@ def time_visual_compress(wl, dev, stream, capture):
             "device_status": sfv.read_device_status(ws)}
 
 
+def time_fused_acceptance(wl, dev, stream, capture):
+    """The target LM head of the B*(k+1) verified positions fused with the
+    acceptance (sf_verify_lm_head_accept) against the two calls it replaces
+    (sf_lm_head, then sf_accept on its logits), over a random bf16 LM head
+    of the target's shape; graphs of 10 calls."""
+    import torch
+    from paper_2505_12728_gb300 import specflash_verify as sfv
+    from paper_2505_12728_gb300.workloads import make_accept_inputs, make_draft_tail_case
+    if wl.B * (wl.k + 1) > 256:
+        return None
+    from paper_2505_12728_gb300.workloads import HIDDEN_SIZES
+    R, d, V = wl.B * (wl.k + 1), HIDDEN_SIZES[wl.V], wl.V
+    case = make_draft_tail_case(R, d, V, seed=[wl.seed, 0xF05E], logit_std=wl.logit_std)
+    acc = make_accept_inputs(wl)
+    bf = lambda bits: torch.from_numpy(np.ascontiguousarray(bits).view(np.int16)).to(dev).view(
+        torch.bfloat16)
+    h, w = bf(case.hidden).view(wl.B, wl.k + 1, d), bf(case.weight)
+    q = torch.from_numpy(acc.draft_probs).to(dev)
+    t = torch.from_numpy(acc.draft_tokens).to(dev)
+    u = torch.from_numpy(acc.uniforms).to(dev)
+    tau = torch.from_numpy(acc.temperature).to(dev)
+    logits = torch.empty((wl.B, wl.k + 1, V), dtype=torch.float32, device=dev)
+    n = torch.empty(wl.B, dtype=torch.int32, device=dev)
+    toks = torch.empty((wl.B, wl.k + 1), dtype=torch.int32, device=dev)
+    ratio = torch.empty((wl.B, wl.k), dtype=torch.float32, device=dev)
+    ws_f = sfv.new_workspace(sfv.verify_lm_head_accept_workspace_size(wl.B, wl.k, V), dev)
+    ws_l = sfv.new_workspace(sfv.draft_tail_workspace_size(R, V), dev)
+    ws_a = sfv.new_workspace(sfv.accept_workspace_size(wl.B, wl.k, V), dev)
+    fused = lambda: sfv.verify_lm_head_accept(h, w, q, t, u, tau, logits=logits, num_accepted=n,
+                                              out_tokens=toks, accept_ratio=ratio, workspace=ws_f,
+                                              stream=stream)
+
+    def unfused():
+        sfv.lm_head(h.view(R, d), w, logits=logits.view(R, V), workspace=ws_l, stream=stream)
+        sfv.accept(logits, q, t, u, tau, num_accepted=n, out_tokens=toks, accept_ratio=ratio,
+                   workspace=ws_a, stream=stream)
+
+    def per_call_us(fn, calls=10, reps=5):
+        fn()
+        g = capture(lambda: [fn() for _ in range(calls)])
+        g.replay()
+        a = torch.cuda.Event(enable_timing=True)
+        b = torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        for _ in range(reps):
+            g.replay()
+        b.record(stream)
+        torch.cuda.synchronize()
+        return a.elapsed_time(b) * 1e3 / (calls * reps)
+
+    fused_us = per_call_us(fused)
+    n_f = n.clone()
+    unfused_us = per_call_us(unfused)
+    return {"rows": R, "hidden": d, "vocab": V, "fused_us": fused_us, "unfused_us": unfused_us,
+            "same_num_accepted": bool(torch.equal(n_f, n)),
+            "device_status": sfv.read_device_status(ws_f)}
+
+
 def workload_config(wl, seq_lens):
     return {"workload": wl.name, "description": wl.description, "batch": wl.B,
             "layers": wl.layers, "H_q": wl.H_q, "H_kv": wl.H_kv, "head_dim": wl.d,
@@ -560,6 +618,7 @@ def run_ours(args):
     # B*k draft rows that produce q and T'; outside the verification step)
     dt = time_draft_tail(wl, dev, stream, capture) if not args.no_draft_tail else None
     vcomp = time_visual_compress(wl, dev, stream, capture) if not args.no_draft_tail else None
+    fused_acc = time_fused_acceptance(wl, dev, stream, capture) if not args.no_draft_tail else None
 
     # ---- end to end through host buffers ----
     pin = lambda a: torch.from_numpy(np.ascontiguousarray(a)).pin_memory()
@@ -628,6 +687,7 @@ def run_ours(args):
         "kv_commit_us": commit_us,
         "draft_tail": dt,
         "visual_compress": vcomp,
+        "lm_head_accept": fused_acc,
         "mean_accepted": float(n_acc.float().mean().item()),
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                      "frac": achieved / peak,
@@ -669,7 +729,8 @@ def main(argv=None):
                     help="seconds of oracle work for the cpu_baseline sample")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-draft-tail", action="store_true",
-                    help="skip the draft-side timings (LM head + sampling, visual compressor)")
+                    help="skip the draft-side and LM-head timings (draft tail, visual compressor, "
+                         "fused target LM head + acceptance)")
     ap.add_argument("--eager", action="store_true",
                     help="launch every call from Python instead of replaying CUDA graphs")
     args = ap.parse_args(argv)
