@@ -35,6 +35,7 @@
 // float-float gives the accuracy the decisions need.
 #include <climits>
 #include <cmath>
+#include <mutex>
 
 #include "ff_math.cuh"
 #include "sf_device.cuh"
@@ -301,6 +302,324 @@ accept_stats_kernel(const __grid_constant__ AccParams p) {
   __syncthreads();
   decide_sequence(p, b, greedy, tau, my_tok, my_u, s_rm, s_rarg, s_rS, s_rlx, s_rqx, s_rhx, s_acc);
   if (tid == 0) p.seq_tickets[b] = 0u;
+}
+
+// Single-kernel acceptance for V <= 16 * kClusterMaxSlice: one thread-block
+// cluster of cs CTAs per sequence, CTA `rank` owning tokens [rank * slice,
+// (rank + 1) * slice) of every row.  Phases, separated by cluster barriers
+// (the same number on every path; greedy clusters leave together after the
+// decision):
+//  1. each warp reduces one row of the CTA's slice to (max, first argmax,
+//     float-float sum of exp((x - max)/tau));
+//  2. CTA 0 combines the cs records of each row (read through distributed
+//     shared memory, in rank order), takes the decisions (decide_sequence)
+//     and publishes j and row j's (max, sum);
+//  3. sampled sequences: each CTA writes row j's residual (or bonus) terms
+//     of its slice to shared memory and their ordered sum;
+//  4. every CTA adds the cs slice sums in rank order, finds the slice
+//     holding u_k * S, and that CTA scans its terms in ascending order.
+constexpr int kClusterMax = 16;
+constexpr int kClusterMaxSlice = 2048;   // tokens per CTA: one row slice in a warp's registers
+constexpr int kClusterPerThread = kClusterMaxSlice / kAccThreads;  // 8
+
+struct alignas(16) ClusterRec {  // one row of one CTA's slice (one 16-byte remote load)
+  float m;
+  int arg;
+  ff S;
+};
+
+struct alignas(16) ClusterDraw {  // row j's terms in one CTA's slice (two 16-byte loads)
+  ff sum_r, sum_p;
+  int last_r, last_p;
+  int pad[2];
+};
+static_assert(sizeof(ClusterRec) == 16 && sizeof(ClusterDraw) == 32, "record sizes");
+
+__global__ void __launch_bounds__(kAccThreads)
+accept_cluster_kernel(const __grid_constant__ AccParams p, int cs, int slice) {
+  extern __shared__ float s_terms[];  // [slice]
+  __shared__ ClusterRec s_rec[SF_MAX_DRAFT + 1];
+  __shared__ ClusterRec s_part[SF_MAX_DRAFT + 1][kAccWarps];  // per-warp partials of phase 1
+  __shared__ ClusterDraw s_draw;
+  __shared__ int s_dec_j;
+  __shared__ float s_dec_m;
+  __shared__ ff s_dec_S;
+  __shared__ ff s_d[32];
+  __shared__ ff s_scan[kAccWarps + 1];
+  __shared__ int s_acc[SF_MAX_DRAFT];
+  __shared__ float s_rm[SF_MAX_DRAFT + 1], s_rlx[SF_MAX_DRAFT + 1], s_rqx[SF_MAX_DRAFT + 1];
+  __shared__ int s_rarg[SF_MAX_DRAFT + 1], s_rhx[SF_MAX_DRAFT + 1];
+  __shared__ ff s_rS[SF_MAX_DRAFT + 1];
+  __shared__ int s_i0, s_i1;
+  __shared__ ff s_base, s_total;
+
+  grid_dependency_wait();  // logits, q, tokens and the outputs follow the previous kernel
+  grid_launch_dependents();
+  const int rank = blockIdx.x, b = blockIdx.y;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int k = p.k, V = p.V;
+  const float tau = p.tau[b];
+  const bool greedy = !(tau > 0.0f);
+  const int x0 = min(V, rank * slice), x1 = min(V, x0 + slice);
+
+  // ---- 1. row statistics of the slice: warp w reduces the w-th eighth of
+  // the slice of every row (rows interleaved, short dependency chains), then
+  // warp r merges row r's eight partials in warp order ----
+  {
+    constexpr int kRG = 6;  // rows per pass
+    const int sub = kClusterMaxSlice / kAccWarps;  // 256 tokens per warp
+    const int w0 = x0 + warp * sub, w1 = min(x1, w0 + sub);
+    for (int g = 0; g <= k; g += kRG) {
+      float v[kRG][8];
+#pragma unroll
+      for (int i = 0; i < kRG; ++i) {
+        const int r = g + i;
+        const float *row = p.logits + ((size_t)b * (k + 1) + (r <= k ? r : k)) * V;
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+          const int e = w0 + 4 * (lane + 32 * h);
+          float4 x = make_float4(-INFINITY, -INFINITY, -INFINITY, -INFINITY);
+          if (r <= k) {
+            if (p.vec4) {
+              if (e < w1) x = *reinterpret_cast<const float4 *>(row + e);
+            } else {
+              if (e < w1) x.x = row[e];
+              if (e + 1 < w1) x.y = row[e + 1];
+              if (e + 2 < w1) x.z = row[e + 2];
+              if (e + 3 < w1) x.w = row[e + 3];
+            }
+          }
+          v[i][4 * h] = x.x; v[i][4 * h + 1] = x.y; v[i][4 * h + 2] = x.z; v[i][4 * h + 3] = x.w;
+        }
+      }
+#pragma unroll
+      for (int i = 0; i < kRG; ++i) {
+        float bv = -INFINITY;
+        int bi = INT_MAX;
+#pragma unroll
+        for (int t = 0; t < 8; ++t) {
+          const int e = w0 + 4 * (lane + 32 * (t / 4)) + (t % 4);
+          if (better(v[i][t], e, bv, bi)) { bv = v[i][t]; bi = e; }
+        }
+        warp_argmax(bv, bi);
+        ff S = ff_of(0.f);
+        if (!greedy && bv != -INFINITY) {
+#pragma unroll
+          for (int t = 0; t < 8; ++t)
+            if (v[i][t] != -INFINITY) S = ff_add(S, ff_of(exp_scaled(v[i][t], bv, tau)));
+          S = warp_sum_ff(S);
+        }
+        if (lane == 0 && g + i <= k) s_part[g + i][warp] = ClusterRec{bv, bi, S};
+      }
+    }
+    __syncthreads();
+    for (int r = warp; r <= k; r += kAccWarps) {
+      // lane w < 8 holds warp w's partial; merged in warp order
+      float cm = -INFINITY;
+      int ca = INT_MAX;
+      ff cS = ff_of(0.f);
+      if (lane < kAccWarps) {
+        cm = s_part[r][lane].m;
+        ca = s_part[r][lane].arg;
+        cS = s_part[r][lane].S;
+      }
+      float mv = cm;
+      int mi = ca;
+      warp_argmax(mv, mi);
+      ff Sr = ff_of(0.f);
+      if (!greedy && mv != -INFINITY) {
+        for (int w = 0; w < kAccWarps; ++w) {
+          const float wm = __shfl_sync(0xffffffffu, cm, w);
+          const ff wS = ff{__shfl_sync(0xffffffffu, cS.hi, w), __shfl_sync(0xffffffffu, cS.lo, w)};
+          if (ff_pos(wS)) Sr = ff_add(Sr, ff_mul(wS, exp_diff_accurate(wm, mv, tau)));
+        }
+      }
+      if (lane == 0) s_rec[r] = ClusterRec{mv, mi, Sr};
+    }
+  }
+  cluster_sync();
+
+  // ---- 2. CTA 0: combine the slices of every row and decide ----
+  if (rank == 0) {
+    int my_tok = -1;
+    float my_u = 0.f;
+    if (tid < k) {
+      my_tok = p.tokens[(size_t)b * k + tid];
+      my_u = p.u[(size_t)b * (k + 1) + tid];
+    }
+    for (int r = warp; r <= k; r += kAccWarps) {
+      float mv = -INFINITY, cm = -INFINITY;
+      int mi = INT_MAX;
+      ff cS = ff_of(0.f);
+      if (lane < cs) {
+        const float4 rec = ld_dsmem_f32x4(smem_addr(&s_rec[r]), lane);
+        cm = rec.x;
+        cS = ff{rec.z, rec.w};
+        mv = cm;
+        mi = __float_as_int(rec.y);
+      }
+      warp_argmax(mv, mi);
+      ff Sr = ff_of(0.f);
+      if (!greedy && mv != -INFINITY) {
+        if (lane < cs && ff_pos(cS)) Sr = ff_mul(cS, exp_diff_accurate(cm, mv, tau));
+        Sr = warp_sum_ff(Sr);
+      }
+      if (lane == 0) {
+        const int x = r < k ? p.tokens[(size_t)b * k + r] : -1;
+        const bool ok = x >= 0 && x < V;
+        s_rm[r] = mv;
+        s_rarg[r] = mi;
+        s_rS[r] = Sr;
+        s_rlx[r] = ok ? p.logits[((size_t)b * (k + 1) + r) * V + x] : 0.f;
+        s_rqx[r] = ok ? p.q[((size_t)b * k + r) * V + x] : 0.f;
+        s_rhx[r] = ok ? 1 : 0;
+      }
+    }
+    __syncthreads();
+    decide_sequence(p, b, greedy, tau, my_tok, my_u, s_rm, s_rarg, s_rS, s_rlx, s_rqx, s_rhx, s_acc);
+    // publish j and row j's (max, sum) into every CTA's shared memory
+    if (tid < cs) {
+      int j = k;
+      for (int i = 0; i < k; ++i)
+        if (!s_acc[i]) { j = i; break; }
+      st_dsmem_f32(dsmem_addr(smem_addr(&s_dec_j), tid), __int_as_float(j));
+      st_dsmem_f32(dsmem_addr(smem_addr(&s_dec_m), tid), s_rm[j]);
+      st_dsmem_f32(dsmem_addr(smem_addr(&s_dec_S), tid), s_rS[j].hi);
+      st_dsmem_f32(dsmem_addr(smem_addr(&s_dec_S) + 4, tid), s_rS[j].lo);
+    }
+  }
+  cluster_sync();
+  if (greedy) return;  // uniform over the cluster: the sequence is complete
+
+  // ---- 3. row j's residual (or bonus) terms of the slice ----
+  const int j = s_dec_j;
+  const float mj = s_dec_m;
+  const ff Sj = s_dec_S;
+  const bool residual = j < k;
+  const float invS = ff_div_to_f(1.0f, Sj);
+  const float *row = p.logits + ((size_t)b * (k + 1) + j) * V;
+  const float *qrow = residual ? p.q + ((size_t)b * k + j) * V : nullptr;
+  const int len = x1 - x0;
+  ff sp = ff_of(0.f);
+  int lr = -1, lp = -1;
+  {
+    float xv[kClusterPerThread], qv[kClusterPerThread];
+#pragma unroll
+    for (int t = 0; t < kClusterPerThread; ++t) {
+      const int e = tid + kAccThreads * t;
+      xv[t] = e < len ? row[x0 + e] : 0.f;
+      qv[t] = (residual && e < len) ? qrow[x0 + e] : 0.f;
+    }
+#pragma unroll
+    for (int t = 0; t < kClusterPerThread; ++t) {
+      const int e = tid + kAccThreads * t;
+      if (e < len) {
+        float rr, pz;
+        draw_terms(xv[t], qv[t], residual, mj, tau, invS, rr, pz);
+        s_terms[e] = rr;
+        sp = ff_add(sp, ff_of(pz));
+        if (rr > 0.f) lr = x0 + e;
+        if (pz > 0.f) lp = x0 + e;
+      }
+    }
+  }
+  __syncthreads();
+  // thread t owns the contiguous run [a0, a1) of the slice, summed in order
+  const int per = (len + kAccThreads - 1) / kAccThreads;
+  const int a0 = min(len, tid * per), a1 = min(len, a0 + per);
+  {
+    ff mine = ff_of(0.f);
+    for (int e = a0; e < a1; ++e) mine = ff_add(mine, ff_of(s_terms[e]));
+    ff ex, tot;
+    block_inclusive_scan(mine, s_scan, &ex, &tot);
+    const ff tp = block_sum(sp, s_d);
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      lr = max(lr, __shfl_xor_sync(0xffffffffu, lr, o));
+      lp = max(lp, __shfl_xor_sync(0xffffffffu, lp, o));
+    }
+    if (tid == 0) { s_i0 = -1; s_i1 = -1; }
+    __syncthreads();
+    if (lane == 0) { atomicMax(&s_i0, lr); atomicMax(&s_i1, lp); }
+    __syncthreads();
+    if (tid == 0) s_draw = ClusterDraw{tot, tp, s_i0, s_i1, {0, 0}};
+  }
+  cluster_sync();
+
+  // ---- 4. the slice holding u_k * S draws the token ----
+  if (warp == 0) {
+    // lane l reads slice l's record (all in flight together); the sums run
+    // in rank order through shuffles, identically in every CTA
+    ff r_l = ff_of(0.f), p_l = ff_of(0.f);
+    int lr_l = -1, lp_l = -1;
+    if (lane < cs) {
+      const uint32_t a = smem_addr(&s_draw);
+      const float4 s0 = ld_dsmem_f32x4(a, lane), s1 = ld_dsmem_f32x4(a + 16, lane);
+      r_l = ff{s0.x, s0.y};
+      p_l = ff{s0.z, s0.w};
+      lr_l = __float_as_int(s1.x);
+      lp_l = __float_as_int(s1.y);
+    }
+    ff tr = ff_of(0.f), tp = ff_of(0.f);
+    for (int l = 0; l < cs; ++l) {
+      tr = ff_add(tr, ff{__shfl_sync(0xffffffffu, r_l.hi, l), __shfl_sync(0xffffffffu, r_l.lo, l)});
+      tp = ff_add(tp, ff{__shfl_sync(0xffffffffu, p_l.hi, l), __shfl_sync(0xffffffffu, p_l.lo, l)});
+    }
+    const bool use_p = !ff_pos(tr);  // residual with no mass (rounding only)
+    const ff total = use_p ? tp : tr;
+    const ff target = ff_mul(total, p.u[(size_t)b * (k + 1) + k]);
+    // slice l covers [cum_l, cum_l + sum_l); cum_{l+1} = ff_add(cum_l, sum_l) exactly
+    int cross = -1, last = -1;
+    ff cum = ff_of(0.f), base = ff_of(0.f);
+    for (int l = 0; l < cs; ++l) {
+      const ff mine = use_p ? p_l : r_l;
+      const ff sl = ff{__shfl_sync(0xffffffffu, mine.hi, l), __shfl_sync(0xffffffffu, mine.lo, l)};
+      const ff nxt = ff_add(cum, sl);
+      last = max(last, __shfl_sync(0xffffffffu, use_p ? lp_l : lr_l, l));
+      if (cross < 0 && ff_pos(sl) && ff_lt(target, nxt) && !ff_lt(target, cum)) {
+        cross = l;
+        base = cum;
+      }
+      cum = nxt;
+    }
+    if (lane == 0) {
+      s_i0 = cross;
+      s_i1 = use_p ? 1 : 0;
+      s_total = target;
+      s_base = base;
+      // no slice holds the target (rounding): the last token with positive mass
+      if (cross < 0 && rank == 0) p.out_tokens[(size_t)b * (k + 1) + j] = last;
+    }
+  }
+  __syncthreads();
+  if (s_i0 == rank) {
+    const bool use_p = s_i1 != 0;
+    if (use_p) {
+      for (int e = tid; e < len; e += kAccThreads) {
+        float rr, pz;
+        draw_terms(row[x0 + e], 0.f, false, mj, tau, invS, rr, pz);
+        s_terms[e] = pz;
+      }
+      __syncthreads();
+    }
+    const ff target = s_total;
+    ff mine = ff_of(0.f);
+    for (int e = a0; e < a1; ++e) mine = ff_add(mine, ff_of(s_terms[e]));
+    ff ex, tot;
+    block_inclusive_scan(mine, s_scan, &ex, &tot);
+    ff c = ff_add(s_base, ex);
+    if (tid == 0) s_i0 = INT_MAX;
+    __syncthreads();
+    for (int e = a0; e < a1; ++e) {
+      c = ff_add(c, ff_of(s_terms[e]));
+      if (ff_lt(target, c)) { atomicMin(&s_i0, x0 + e); break; }
+    }
+    __syncthreads();
+    if (tid == 0)
+      p.out_tokens[(size_t)b * (k + 1) + j] =
+          s_i0 != INT_MAX ? s_i0 : (use_p ? s_draw.last_p : s_draw.last_r);
+  }
+  cluster_sync();  // peers may still read this CTA's s_draw
 }
 
 // Fused path: the decisions from the projection's per-CTA row statistics
@@ -576,6 +895,36 @@ static AccLayout acc_layout(int B, int k, const AccPlan &pl) {
   return l;
 }
 
+// Cluster size and slice of the single-kernel path: up to 16 CTAs per
+// sequence, slices of at most kClusterMaxSlice tokens (a multiple of 4);
+// false when V needs more (the two-kernel path spreads those rows over
+// many more CTAs).
+static bool cluster_plan(int V, int *cs, int *slice) {
+  int c = (V + kClusterMaxSlice - 1) / kClusterMaxSlice;
+  if (c > kClusterMax) c = kClusterMax;
+  if (c < 1) c = 1;
+  int sl = (V + c - 1) / c;
+  sl = (sl + 3) / 4 * 4;
+  if (sl > kClusterMaxSlice) return false;
+  *cs = c;
+  *slice = sl;
+  return true;
+}
+
+static int cluster_setup() {
+  static std::once_flag once;
+  static cudaError_t err = cudaSuccess;
+  std::call_once(once, [] {
+    err = cudaFuncSetAttribute(accept_cluster_kernel, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+    if (err == cudaSuccess)
+      err = cudaFuncSetAttribute(accept_cluster_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 static_cast<int>(sizeof(float) * kClusterMaxSlice));
+  });
+  if (err != cudaSuccess)
+    return fail(SF_ERR_CUDA, "cudaFuncSetAttribute (accept cluster): %s", cudaGetErrorString(err));
+  return SF_OK;
+}
+
 static int check_accept_shapes(int B, int k, int V) {
   if (B < 1 || B > SF_MAX_BATCH) return fail(SF_ERR_INVALID_ARG, "B=%d outside [1, %d]", B, SF_MAX_BATCH);
   if (k < 1 || k > SF_MAX_DRAFT) return fail(SF_ERR_INVALID_ARG, "k=%d outside [1, %d]", k, SF_MAX_DRAFT);
@@ -645,6 +994,30 @@ int sf_accept(const float *target_logits, const float *draft_probs,
   prm.C2 = plan.C2;
   prm.CV2 = plan.CV2;
   prm.vec4 = (V % 4 == 0) && aligned(target_logits, 16) && aligned(draft_probs, 16);
+
+  // One cluster per sequence when a row fits 16 slices: a single launch
+  int cs = 0, slice = 0;
+  if (cluster_plan(V, &cs, &slice)) {
+    st = cluster_setup();
+    if (st != SF_OK) return st;
+    cudaLaunchAttribute cattr[2];
+    cattr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    cattr[0].val.programmaticStreamSerializationAllowed = 1;
+    cattr[1].id = cudaLaunchAttributeClusterDimension;
+    cattr[1].val.clusterDim.x = cs;
+    cattr[1].val.clusterDim.y = 1;
+    cattr[1].val.clusterDim.z = 1;
+    cudaLaunchConfig_t ccfg = {};
+    ccfg.gridDim = dim3(cs, B);
+    ccfg.blockDim = dim3(kAccThreads);
+    ccfg.dynamicSmemBytes = sizeof(float) * slice;
+    ccfg.stream = stream;
+    ccfg.attrs = cattr;
+    ccfg.numAttrs = 2;
+    cudaError_t ce = cudaLaunchKernelEx(&ccfg, accept_cluster_kernel, prm, cs, slice);
+    if (ce != cudaSuccess) return fail(SF_ERR_CUDA, "accept cluster launch: %s", cudaGetErrorString(ce));
+    return SF_OK;
+  }
 
   // Both kernels are launched with programmatic stream serialisation: each
   // may be scheduled while the previous kernel on the stream drains and

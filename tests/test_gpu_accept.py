@@ -55,6 +55,12 @@ def test_many_sequences_match_oracle(oracle_mod, V):
     _check(oracle_mod, inp)
 
 
+@pytest.mark.parametrize("mode", ["sampling", "greedy", "alternate"])
+def test_vocabulary_beyond_the_single_kernel_path(oracle_mod, mode):
+    # V above 16 slices of 2048 tokens: the two-kernel (statistics, draw) path
+    _check(oracle_mod, make_accept_case(3, 4, 200003, seed=17, mode=mode))
+
+
 @pytest.mark.parametrize("V,k", [(2, 3), (3, 2), (5, 2), (5, 3)])
 def test_brute_force_tiny_vocabularies(oracle_mod, V, k):
     # Every draft tuple in [0, V)^k, each with 64 uniform vectors drawn from
