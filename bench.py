@@ -550,38 +550,47 @@ def run_ours(args):
 
     use_graph = not args.eager
     if use_graph:
+        # the step as one graph (the timed quantity), and its two parts as
+        # separate graphs for the per-part breakdown
+        g_step = capture(step)
         g_att = capture(lambda: attention_layers(q))
         g_acc = capture(lambda: acceptance(logits, qprob, toks, uni, temp))
-        run_att, run_acc = g_att.replay, g_acc.replay
+        run_step, run_att, run_acc = g_step.replay, g_att.replay, g_acc.replay
     else:
+        run_step = step
         run_att = lambda: attention_layers(q)
         run_acc = lambda: acceptance(logits, qprob, toks, uni, temp)
     # clocks are sampled from the warm-up through the end of the timed region
     clocks = ClockSampler(local)
     clocks.start()
     for _ in range(args.warmup):
-        run_att()
-        run_acc()
+        run_step()
     torch.cuda.synchronize()
 
-    # ---- device-resident timing ----
-    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(args.steps)]
+    # ---- device-resident timing: K steps back to back ----
     barrier(world)
     torch.cuda.synchronize()
     t_start = torch.cuda.Event(enable_timing=True)
     t_end = torch.cuda.Event(enable_timing=True)
     t_start.record(stream)
+    for _ in range(args.steps):
+        run_step()
+    t_end.record(stream)
+    torch.cuda.synchronize()
+    barrier(world)
+    clk = clocks.stop()
+    total_ms = max_over_ranks(t_start.elapsed_time(t_end), world, dev)
+
+    # ---- per-part breakdown (the two parts as separate launches, with
+    # events between them; the part boundary costs a launch here) ----
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(args.steps)]
     for s in range(args.steps):
         ev[s][0].record(stream)
         run_att()
         ev[s][1].record(stream)
         run_acc()
         ev[s][2].record(stream)
-    t_end.record(stream)
     torch.cuda.synchronize()
-    barrier(world)
-    clk = clocks.stop()
-    total_ms = max_over_ranks(t_start.elapsed_time(t_end), world, dev)
     att_ms = [ev[s][0].elapsed_time(ev[s][1]) for s in range(args.steps)]
     acc_ms = [ev[s][1].elapsed_time(ev[s][2]) for s in range(args.steps)]
     ms_per_step = total_ms / args.steps
