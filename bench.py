@@ -629,30 +629,43 @@ def run_ours(args):
     vcomp = time_visual_compress(wl, dev, stream, capture) if not args.no_draft_tail else None
     fused_acc = time_fused_acceptance(wl, dev, stream, capture) if not args.no_draft_tail else None
 
-    # ---- end to end through host buffers ----
-    pin = lambda a: torch.from_numpy(np.ascontiguousarray(a)).pin_memory()
-    h_q = pin(att.q.view(np.int16))
-    h_logits, h_qprob = pin(acc.target_logits), pin(acc.draft_probs)
-    h_toks, h_uni, h_temp = pin(acc.draft_tokens), pin(acc.uniforms), pin(acc.temperature)
-    h_n = torch.empty(wl.B, dtype=torch.int32).pin_memory()
-    h_out = torch.empty((wl.B, wl.k + 1), dtype=torch.int32).pin_memory()
-    d_q = torch.empty_like(q)
-    d_logits, d_qprob = torch.empty_like(logits), torch.empty_like(qprob)
-    d_toks, d_uni, d_temp = torch.empty_like(toks), torch.empty_like(uni), torch.empty_like(temp)
-    h2d = sum(t.numel() * t.element_size() for t in (h_q, h_logits, h_qprob, h_toks, h_uni, h_temp))
-    d2h = h_n.numel() * 4 + h_out.numel() * 4
+    # ---- end to end through host buffers: the step's inputs are packed in
+    # one pinned staging buffer (one host-to-device copy per step) and its
+    # results in one device buffer (one device-to-host copy) ----
+    inputs = [att.q.view(np.int16), acc.target_logits, acc.draft_probs, acc.draft_tokens,
+              acc.uniforms, acc.temperature]
+    offs, total = [], 0
+    for a in inputs:
+        offs.append(total)
+        total += (a.nbytes + 255) // 256 * 256
+    h_stage = torch.empty(total, dtype=torch.uint8).pin_memory()
+    for a, o in zip(inputs, offs):
+        h_stage[o:o + a.nbytes].copy_(torch.from_numpy(np.ascontiguousarray(a).view(np.uint8).reshape(-1)))
+    d_stage = torch.empty(total, dtype=torch.uint8, device=dev)
+
+    def staged(i, dtype, shape):
+        n = inputs[i].nbytes
+        return d_stage[offs[i]:offs[i] + n].view(dtype).view(shape)
+
+    d_q = staged(0, torch.bfloat16, tuple(q.shape))
+    d_logits = staged(1, torch.float32, tuple(logits.shape))
+    d_qprob = staged(2, torch.float32, tuple(qprob.shape))
+    d_toks = staged(3, torch.int32, tuple(toks.shape))
+    d_uni = staged(4, torch.float32, tuple(uni.shape))
+    d_temp = staged(5, torch.float32, tuple(temp.shape))
+    d_res = torch.empty(wl.B * (wl.k + 2), dtype=torch.int32, device=dev)
+    e_n, e_out = d_res[:wl.B], d_res[wl.B:].view(wl.B, wl.k + 1)
+    h_res = torch.empty(wl.B * (wl.k + 2), dtype=torch.int32).pin_memory()
+    h_n, h_out = h_res[:wl.B], h_res[wl.B:].view(wl.B, wl.k + 1)
+    h2d = h_stage.numel()  # the packed inputs (each padded to 256 bytes)
+    d2h = h_res.numel() * 4
 
     def e2e_step():
-        d_q.view(torch.int16).copy_(h_q, non_blocking=True)
-        d_logits.copy_(h_logits, non_blocking=True)
-        d_qprob.copy_(h_qprob, non_blocking=True)
-        d_toks.copy_(h_toks, non_blocking=True)
-        d_uni.copy_(h_uni, non_blocking=True)
-        d_temp.copy_(h_temp, non_blocking=True)
+        d_stage.copy_(h_stage, non_blocking=True)
         attention_layers(d_q)
-        acceptance(d_logits, d_qprob, d_toks, d_uni, d_temp)
-        h_n.copy_(n_acc, non_blocking=True)
-        h_out.copy_(out_toks, non_blocking=True)
+        sfv.accept(d_logits, d_qprob, d_toks, d_uni, d_temp, num_accepted=e_n, out_tokens=e_out,
+                   accept_ratio=ratio, workspace=ws_acc, stream=stream)
+        h_res.copy_(d_res, non_blocking=True)
 
     for _ in range(args.warmup):
         e2e_step()
