@@ -911,17 +911,41 @@ static bool cluster_plan(int V, int *cs, int *slice) {
   return true;
 }
 
-static int cluster_setup() {
-  static std::once_flag once;
-  static cudaError_t err = cudaSuccess;
-  std::call_once(once, [] {
-    err = cudaFuncSetAttribute(accept_cluster_kernel, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
-    if (err == cudaSuccess)
-      err = cudaFuncSetAttribute(accept_cluster_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 static_cast<int>(sizeof(float) * kClusterMaxSlice));
-  });
-  if (err != cudaSuccess)
-    return fail(SF_ERR_CUDA, "cudaFuncSetAttribute (accept cluster): %s", cudaGetErrorString(err));
+// Sets the kernel attributes once per device and reports whether a cluster
+// of cs CTAs can be resident (*ok false: use the two-kernel path).
+static int cluster_setup(int cs, bool *ok) {
+  static std::mutex mu;
+  static int state[64][kClusterMax + 1] = {};  // 0 unknown, 1 usable, 2 not usable
+  DeviceInfo dev;
+  int st = current_device(&dev);
+  if (st != SF_OK) return st;
+  if (dev.ordinal < 0 || dev.ordinal >= 64) return fail(SF_ERR_UNSUPPORTED, "device ordinal %d", dev.ordinal);
+  std::lock_guard<std::mutex> lock(mu);
+  if (state[dev.ordinal][cs] == 0) {
+    cudaError_t e = cudaFuncSetAttribute(accept_cluster_kernel,
+                                         cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+    if (e == cudaSuccess)
+      e = cudaFuncSetAttribute(accept_cluster_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                               static_cast<int>(sizeof(float) * kClusterMaxSlice));
+    if (e != cudaSuccess)
+      return fail(SF_ERR_CUDA, "cudaFuncSetAttribute (accept cluster): %s", cudaGetErrorString(e));
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = cs;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(cs, 1);
+    cfg.blockDim = dim3(kAccThreads);
+    cfg.dynamicSmemBytes = sizeof(float) * kClusterMaxSlice;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    int n = 0;
+    e = cudaOccupancyMaxActiveClusters(&n, accept_cluster_kernel, &cfg);
+    if (e != cudaSuccess) (void)cudaGetLastError();  // not usable: clear the error
+    state[dev.ordinal][cs] = (e == cudaSuccess && n > 0) ? 1 : 2;
+  }
+  *ok = state[dev.ordinal][cs] == 1;
   return SF_OK;
 }
 
@@ -997,9 +1021,12 @@ int sf_accept(const float *target_logits, const float *draft_probs,
 
   // One cluster per sequence when a row fits 16 slices: a single launch
   int cs = 0, slice = 0;
+  bool cluster_ok = false;
   if (cluster_plan(V, &cs, &slice)) {
-    st = cluster_setup();
+    st = cluster_setup(cs, &cluster_ok);
     if (st != SF_OK) return st;
+  }
+  if (cluster_ok) {
     cudaLaunchAttribute cattr[2];
     cattr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
     cattr[0].val.programmaticStreamSerializationAllowed = 1;
