@@ -101,9 +101,16 @@ struct AccParams {
 };
 
 
+// exp((x - m) / tau) for the per-token loops (sums and draw terms); the
+// decisions' p(x) use exp_diff_accurate.  Terms are summed four at a time in
+// fp32 before each float-float add (a few 2^-24 of the partial).
 __device__ __forceinline__ float exp_scaled(float x, float m, float tau) {
   const float d = __fsub_rn(x, m);
-  return expf(tau == 1.0f ? d : __fdiv_rn(d, tau));
+  return exp_fast(tau == 1.0f ? d : __fdiv_rn(d, tau));
+}
+
+__device__ __forceinline__ float sum4(float a, float b, float c, float d) {
+  return __fadd_rn(__fadd_rn(a, b), __fadd_rn(c, d));
 }
 
 // Residual (j < k) or bonus (j == k) mass of one token and its target mass.
@@ -242,8 +249,14 @@ accept_stats_kernel(const __grid_constant__ AccParams p) {
   if (!greedy && bv != -INFINITY) {
     ff acc = ff_of(0.f);
 #pragma unroll
-    for (int t = 0; t < kMaxPerThread; ++t)
-      if (t < n) acc = ff_add(acc, ff_of(exp_scaled(vals[t], bv, tau)));
+    for (int t = 0; t < kMaxPerThread; t += 4) {
+      if (t < n) {
+        float e[4];
+#pragma unroll
+        for (int u = 0; u < 4; ++u) e[u] = t + u < n ? exp_scaled(vals[t + u], bv, tau) : 0.f;
+        acc = ff_add(acc, ff_of(sum4(e[0], e[1], e[2], e[3])));
+      }
+    }
     S = block_sum(acc, s_d);
   }
 
@@ -404,9 +417,10 @@ accept_cluster_kernel(const __grid_constant__ AccParams p, int cs, int slice) {
         warp_argmax(bv, bi);
         ff S = ff_of(0.f);
         if (!greedy && bv != -INFINITY) {
+          float e[8];
 #pragma unroll
-          for (int t = 0; t < 8; ++t)
-            if (v[i][t] != -INFINITY) S = ff_add(S, ff_of(exp_scaled(v[i][t], bv, tau)));
+          for (int t = 0; t < 8; ++t) e[t] = v[i][t] != -INFINITY ? exp_scaled(v[i][t], bv, tau) : 0.f;
+          S = ff_add(ff_of(sum4(e[0], e[1], e[2], e[3])), ff_of(sum4(e[4], e[5], e[6], e[7])));
           S = warp_sum_ff(S);
         }
         if (lane == 0 && g + i <= k) s_part[g + i][warp] = ClusterRec{bv, bi, S};
@@ -510,18 +524,22 @@ accept_cluster_kernel(const __grid_constant__ AccParams p, int cs, int slice) {
       xv[t] = e < len ? row[x0 + e] : 0.f;
       qv[t] = (residual && e < len) ? qrow[x0 + e] : 0.f;
     }
+    float pzs[kClusterPerThread];
 #pragma unroll
     for (int t = 0; t < kClusterPerThread; ++t) {
       const int e = tid + kAccThreads * t;
+      pzs[t] = 0.f;
       if (e < len) {
-        float rr, pz;
-        draw_terms(xv[t], qv[t], residual, mj, tau, invS, rr, pz);
+        float rr;
+        draw_terms(xv[t], qv[t], residual, mj, tau, invS, rr, pzs[t]);
         s_terms[e] = rr;
-        sp = ff_add(sp, ff_of(pz));
         if (rr > 0.f) lr = x0 + e;
-        if (pz > 0.f) lp = x0 + e;
+        if (pzs[t] > 0.f) lp = x0 + e;
       }
     }
+#pragma unroll
+    for (int t = 0; t < kClusterPerThread; t += 4)
+      sp = ff_add(sp, ff_of(sum4(pzs[t], pzs[t + 1], pzs[t + 2], pzs[t + 3])));
   }
   __syncthreads();
   // thread t owns the contiguous run [a0, a1) of the slice, summed in order
@@ -712,15 +730,15 @@ accept_draw_kernel(const __grid_constant__ AccParams p) {
                                  : make_float4(0.f, 0.f, 0.f, 0.f);
       const float xs[4] = {x.x, x.y, x.z, x.w};
       const float qs[4] = {qv.x, qv.y, qv.z, qv.w};
+      float rr[4], pz[4];
 #pragma unroll
       for (int t = 0; t < 4; ++t) {
-        float rr, pz;
-        draw_terms(xs[t], qs[t], residual, rs.m, tau, invS, rr, pz);
-        sr = ff_add(sr, ff_of(rr));
-        sp = ff_add(sp, ff_of(pz));
-        if (rr > 0.f) lr = e + t;
-        if (pz > 0.f) lp = e + t;
+        draw_terms(xs[t], qs[t], residual, rs.m, tau, invS, rr[t], pz[t]);
+        if (rr[t] > 0.f) lr = e + t;
+        if (pz[t] > 0.f) lp = e + t;
       }
+      sr = ff_add(sr, ff_of(sum4(rr[0], rr[1], rr[2], rr[3])));
+      sp = ff_add(sp, ff_of(sum4(pz[0], pz[1], pz[2], pz[3])));
     }
   } else {
     for (int e = c0 + tid; e < c1; e += kAccThreads) {

@@ -55,6 +55,16 @@ def test_many_sequences_match_oracle(oracle_mod, V):
     _check(oracle_mod, inp)
 
 
+@pytest.mark.parametrize("V", [32000, 152064])
+def test_masked_target_logits_match_oracle(oracle_mod, V):
+    # -inf target logits (a masked vocabulary) have probability 0 on both paths
+    inp = make_accept_case(6, 4, V, seed=21, mode="alternate")
+    inp.target_logits[:, :, ::3] = -np.inf
+    inp.target_logits[:, :, 1] = 40.0  # keep a finite maximum
+    ref, n, toks = _check(oracle_mod, inp)
+    assert ((toks == -1) | (toks % 3 != 0)).all()
+
+
 @pytest.mark.parametrize("mode", ["sampling", "greedy", "alternate"])
 def test_vocabulary_beyond_the_single_kernel_path(oracle_mod, mode):
     # V above 16 slices of 2048 tokens: the two-kernel (statistics, draw) path
