@@ -72,6 +72,15 @@ constexpr int kMaxCluster = 16;  // largest cluster launched (non-portable size)
 constexpr int kPrefetchLines = 64;  // block-table lines prefetched for one sequence
 constexpr int kPushSlots = 2;    // rows a CTA merges in push mode (at most)
 
+// The two halves of a cluster barrier phase, for a phase that opens early and
+// closes later (every thread of every CTA of the cluster arrives, then waits).
+__device__ __forceinline__ void cluster_arrive_relaxed() {
+  asm volatile("barrier.cluster.arrive.relaxed.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void cluster_wait_acquire() {
+  asm volatile("barrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+
 template <int D, int KS, int NW, int STAGES>
 __global__ void __launch_bounds__(NW * 32, (NW == 4 ? 2 : 1))
 verify_attention_kernel(const __grid_constant__ CUtensorMap tmap_k,
@@ -152,6 +161,11 @@ verify_attention_kernel(const __grid_constant__ CUtensorMap tmap_k,
     aligned = ((c0 - base) % tb == 0) && (c1 - c0 == tb);
   }
   int seg_b = 0, seg_h = 0;  // the segment of an aligned cluster
+  // Push mode stores into the shared memory of peer CTAs, which must have
+  // started by then: the first barrier phase opens here and closes right
+  // before the push (long since complete by then, so it costs no wait).
+  const bool push_mode = aligned && p.push;
+  if (push_mode) cluster_arrive_relaxed();
 
   const uint64_t policy = l2_policy_evict_first();
   bool waited = false;    // grid_dependency_wait() done
@@ -419,9 +433,15 @@ verify_attention_kernel(const __grid_constant__ CUtensorMap tmap_k,
           (void)mbar_wait_bounded(bar0 + 8 * (x % STAGES), (x / STAGES) & 1u);
       }
       __syncthreads();
-      if (aligned) {  // the cluster's other CTAs expect this CTA's barrier arrivals
+      // the cluster's other CTAs expect this CTA's barrier arrivals, and in
+      // push mode they may still store into its shared memory until the
+      // second phase completes
+      if (push_mode) {
+        cluster_wait_acquire();
         cluster_sync();
-        if (!p.push) cluster_sync();
+      } else if (aligned) {
+        cluster_sync();
+        cluster_sync();
       }
       return;
     }
@@ -516,10 +536,11 @@ verify_attention_kernel(const __grid_constant__ CUtensorMap tmap_k,
       continue;
     }
 
-    if (aligned && p.push) {
+    if (push_mode) {
       // push each partial row into the shared memory of the CTA that merges
       // it: rank rho merges rows [rho*R/cs, (rho+1)*R/cs); entry
       // [row slot][sender rank] holds O (D floats), m, l (stride D + 4)
+      cluster_wait_acquire();  // every peer has started
       const int cs = p.cs, rank = static_cast<int>(blockIdx.x) % cs;
       auto push_row = [&](int r, const float (&oo)[DT][4], int h, float mm, float ll) {
         const int rho = ((r + 1) * cs - 1) / p.R;
@@ -623,10 +644,10 @@ verify_attention_kernel(const __grid_constant__ CUtensorMap tmap_k,
     }
     __syncthreads();
   }
-  if (aligned && p.push) {
+  if (push_mode) {
     // Every peer has pushed its rows; merge this CTA's rows from its own
     // shared memory, in rank order (= tile order).  Nobody reads this CTA's
-    // shared memory, so there is no second barrier.
+    // shared memory, so there is no third phase.
     cluster_sync();
     const int cs = p.cs, rank = static_cast<int>(blockIdx.x) % cs;
     const int R = p.R;
