@@ -27,6 +27,8 @@ struct AttnParams {
   int cs;             // CTAs per cluster of the launch (1: no clusters)
   int push;           // cluster mode: peers push partial rows into the merging CTA
   int push_off;       // byte offset of the push area in dynamic shared memory
+  int bt_off;         // one sequence: byte offset of its block-table row copied to
+                      // dynamic shared memory at entry (0: read from global memory)
   float *partials;    // [G + B * H_kv][R][D + 2]
   int B, n_q, H_q, H_kv, group, R;
   int num_pages, max_pages, max_tokens;

@@ -70,6 +70,7 @@ struct AttnSmem {
 
 constexpr int kMaxCluster = 16;  // largest cluster launched (non-portable size)
 constexpr int kPrefetchLines = 64;  // block-table lines prefetched for one sequence
+constexpr int kBtCacheEntries = 512;  // longest block-table row copied to shared memory
 constexpr int kPushSlots = 2;    // rows a CTA merges in push mode (at most)
 
 // The two halves of a cluster barrier phase, for a phase that opens early and
@@ -116,10 +117,22 @@ verify_attention_kernel(const __grid_constant__ CUtensorMap tmap_k,
   // first K/V copies) runs before grid_dependency_wait(); Q is read and
   // results are written only after it.
   grid_launch_dependents();
-  // one sequence: bring its block-table row toward the SM while seq_lens is
-  // read (the row is needed as soon as the partition is known)
-  if (p.B == 1 && tid < kPrefetchLines && tid * 32 < p.max_pages)
+  // One sequence: its block-table row is needed as soon as the partition is
+  // known.  A short row is loaded now, while seq_lens is read, and kept in
+  // shared memory, so the first copies wait for one global load, not two; a
+  // longer row is brought toward the SM (L2) instead.
+  constexpr int kBtPer = kBtCacheEntries / NTHREADS;
+  int32_t *s_bt = reinterpret_cast<int32_t *>(smem + p.bt_off);
+  int32_t bt_row[kBtPer];
+  if (p.bt_off) {
+#pragma unroll
+    for (int k = 0; k < kBtPer; ++k) {
+      const int i = tid + k * NTHREADS;
+      bt_row[k] = i < p.max_pages ? __ldg(p.block_table + i) : 0;
+    }
+  } else if (p.B == 1 && tid < kPrefetchLines && tid * 32 < p.max_pages) {
     prefetch_l2(p.block_table + tid * 32);
+  }
   if (tid == 0) {
     for (int s = 0; s < STAGES; ++s) mbar_init(bar0 + 8 * s, 1);
     fence_mbar_init();
@@ -127,6 +140,13 @@ verify_attention_kernel(const __grid_constant__ CUtensorMap tmap_k,
     prefetch_tensormap(&tmap_v);
   }
   tile_prefix<NTHREADS>(p, s_prefix, s_len, s_misc + 8);
+  if (p.bt_off) {
+#pragma unroll
+    for (int k = 0; k < kBtPer; ++k) {
+      const int i = tid + k * NTHREADS;
+      if (i < p.max_pages) s_bt[i] = bt_row[k];
+    }
+  }
   __syncthreads();
 
   // The host sizes the grid from an upper bound of the tile count; with more
@@ -208,7 +228,7 @@ verify_attention_kernel(const __grid_constant__ CUtensorMap tmap_k,
     auto fetch_page = [&](int lt, int pg) -> int {
       const int lp = lt * kPagesPerTile + pg;
       if (lp * kPageTokens >= T) return kBeyondEnd;
-      return p.block_table[(size_t)b * p.max_pages + lp];
+      return p.bt_off ? s_bt[lp] : p.block_table[(size_t)b * p.max_pages + lp];
     };
     auto issue = [&](int slot, int pg, int phys) {
       // one page (16 tokens) of K and V into ring slot `slot`; pages past the
@@ -840,13 +860,15 @@ struct AttnPlan {
   int cs;        // CTAs per cluster (1: no clusters)
   int push;      // cluster mode pushes partial rows (few rows per merging CTA)
   int push_off;  // byte offset of the push area in shared memory
+  int bt_off;    // byte offset of the block-table row in shared memory (0: none)
   int tc;        // 1: the tcgen05 kernel (many rows per KV head)
 };
 
 // Largest dynamic shared memory a launch of variant v can ask for: the
 // per-batch arrays at SF_MAX_BATCH plus a full push area.
 static int max_dynamic_smem(const AttnVariant &v) {
-  return v.smem_fixed + 8 * SF_MAX_BATCH + 16 + kPushSlots * kMaxCluster * (128 + 4) * 4;
+  return v.smem_fixed + 8 * SF_MAX_BATCH + 16 + kPushSlots * kMaxCluster * (128 + 4) * 4 + 16 +
+         4 * kBtCacheEntries;
 }
 
 // Per-device, per-kernel launch facts, computed once: the dynamic shared
@@ -925,6 +947,7 @@ static int plan_attention(int B, int n_q, int H_q, int H_kv, int D, int max_page
   plan->smem = plan->v.smem_fixed + 8 * B;
   plan->push = 0;
   plan->push_off = 0;
+  plan->bt_off = 0;
   plan->tc = 0;
   const long long max_tiles =
       (long long)B * H_kv * (((long long)max_pages_per_seq * SF_PAGE_SIZE + kTileTokens - 1) / kTileTokens);
@@ -983,6 +1006,20 @@ static int plan_attention(int B, int n_q, int H_q, int H_kv, int D, int max_page
     plan->push = 1;
     plan->push_off = static_cast<int>(round_up((size_t)plan->v.prefix_off + 4 * (2 * B + 2), 16));
     plan->smem = plan->push_off + 1024 + kPushSlots * plan->cs * (D + 4) * 4;
+  }
+  if (B == 1 && max_pages_per_seq <= kBtCacheEntries) {
+    // the sequence's block-table row, copied at entry, after everything else
+    const int off = static_cast<int>(round_up((size_t)plan->smem - 1024, 16));
+    const int smem = off + 1024 + 4 * max_pages_per_seq;
+    int occ_before = 0, occ_after = 0;
+    st = kernel_setup(plan->v, dev.ordinal, plan->smem, &occ_before);
+    if (st != SF_OK) return st;
+    st = kernel_setup(plan->v, dev.ordinal, smem, &occ_after);
+    if (st != SF_OK) return st;
+    if (occ_after == occ_before) {  // only where it costs no resident CTA
+      plan->bt_off = off;
+      plan->smem = smem;
+    }
   }
   return SF_OK;
 }
@@ -1095,6 +1132,7 @@ int sf_verify_attention(const void *q, const void *k_cache, const void *v_cache,
   prm.cs = plan.cs;
   prm.push = plan.push;
   prm.push_off = plan.push_off;
+  prm.bt_off = plan.bt_off;
   prm.partials = reinterpret_cast<float *>(ws + lay.partials_off);
   prm.B = B;
   prm.n_q = n_q;

@@ -216,3 +216,22 @@ def test_growing_scores_move_the_running_maximum(oracle_mod, n_q, H_q, H_kv):
     for splits in (0, 3):
         out, lse = run_attention(case, num_splits=splits)
         assert_attention_close(out, lse, ref_out, ref_lse)
+
+
+@pytest.mark.parametrize("prefix,max_pages", [
+    (1200, None),   # 76 pages, row of 76 entries: copied to shared memory
+    (1200, 512),    # row of 512 entries (436 unused, -1): copied
+    (1200, 513),    # one entry wider: read from global memory
+    (8187, None),   # 8192 tokens = 512 pages, every entry used: copied
+    (8188, None),   # 513 pages: read from global memory
+])
+def test_one_sequence_block_table_row_widths(oracle_mod, prefix, max_pages):
+    # A single sequence's block-table row of up to 512 entries is copied to
+    # shared memory at kernel entry; wider rows are read from global memory.
+    # Both sides of that limit, with and without unused entries, must give
+    # the oracle's result on the 8-CTA cluster path.
+    case = make_attention_case(1, 5, 32, 32, 128, [prefix], seed=1300 + prefix % 97,
+                               max_pages=max_pages)
+    ref_out, ref_lse = oracle_attention(oracle_mod, case)
+    out, lse = run_attention(case, num_splits=0)
+    assert_attention_close(out, lse, ref_out, ref_lse)
