@@ -181,10 +181,11 @@ accept_stats_kernel(const __grid_constant__ AccParams p) {
   __shared__ int s_rarg[SF_MAX_DRAFT + 1], s_rhx[SF_MAX_DRAFT + 1];
   __shared__ ff s_rS[SF_MAX_DRAFT + 1];
 
-  // The next kernel (the draw) may be scheduled as CTAs of this grid finish.
-  // Inputs are read before grid_dependency_wait() (this library's kernels,
-  // the only ones that let their successor start early, never write them);
-  // the workspace and the outputs are written only after it.
+  // Every input (logits, q, tokens, uniforms, temperatures) may come from
+  // the previous kernel on the stream, which may let this grid start early:
+  // wait for it before reading anything.  Only then let the draw kernel be
+  // scheduled, so that it too starts after the previous kernel completed.
+  grid_dependency_wait();
   grid_launch_dependents();
 
   const int c = blockIdx.x, r = blockIdx.y, b = blockIdx.z;
@@ -260,7 +261,6 @@ accept_stats_kernel(const __grid_constant__ AccParams p) {
     S = block_sum(acc, s_d);
   }
 
-  grid_dependency_wait();  // the workspace and outputs may be in use until here
   const size_t rowid = (size_t)b * (k + 1) + r;
   if (tid == 0) p.chunks[rowid * p.C1 + c] = ChunkRec{bv, bi, S, lx, qx, has_x ? 1 : 0, 0};
 
@@ -699,6 +699,10 @@ accept_draw_kernel(const __grid_constant__ AccParams p) {
   __shared__ int s_flag, s_token, s_chunk, s_last;
   __shared__ ff s_base;
 
+  // The previous kernel (the statistics or decision kernel of this call)
+  // lets this grid start only after it has itself waited for the kernel
+  // before the call, so the call's inputs (temperature, uniforms) are in
+  // place already; j and the row statistics are waited for.
   grid_launch_dependents();
   const int c = blockIdx.x, b = blockIdx.y;
   const int tid = threadIdx.x;

@@ -98,3 +98,32 @@ def test_fused_invalid_arguments():
     assert lib.sf_verify_lm_head_accept_workspace_size(32, 8, 1000) == 0  # 288 rows
     assert lib.sf_verify_lm_head_accept_workspace_size(1, 0, 1000) == 0
     assert lib.sf_verify_lm_head_accept_workspace_size(1, 5, 32000) > 0
+
+
+@pytest.mark.parametrize("V,d", [(152064, 3584), (32000, 4096)])
+def test_lm_head_then_accept_on_one_stream(oracle_mod, V, d):
+    # The target logits written by sf_lm_head are read by sf_accept launched
+    # right after it on the same stream, with no synchronisation between:
+    # the projection lets its successor start early, so the acceptance must
+    # wait for it before reading any input.  The logits buffer is filled with
+    # NaN before each projection, so an early read would show.
+    hidden, weight, inp, ref_logits = make_case(oracle_mod, 4, 8, V, d, seed=[21, V], mode="alternate",
+                                                sharpness=1.5)
+    B, k1, _ = hidden.shape
+    h = bf16_tensor(hidden.reshape(B * k1, d))
+    w = bf16_tensor(weight)
+    dev = {key: torch.from_numpy(getattr(inp, key)).cuda()
+           for key in ("draft_probs", "draft_tokens", "uniforms", "temperature")}
+    logits = torch.empty((B * k1, V), dtype=torch.float32, device="cuda")
+    ws_lm = sfv.new_workspace(sfv.draft_tail_workspace_size(B * k1, V))
+    ws_acc = sfv.new_workspace(sfv.accept_workspace_size(B, k1 - 1, V))
+    ref = oracle_accept(oracle_mod, inp)
+    for _ in range(3):
+        logits.fill_(float("nan"))
+        sfv.lm_head(h, w, logits=logits, workspace=ws_lm)
+        n, toks, ratio = sfv.accept(logits.view(B, k1, V), dev["draft_probs"], dev["draft_tokens"],
+                                    dev["uniforms"], dev["temperature"], workspace=ws_acc)
+        torch.cuda.synchronize()
+        assert np.array_equal(logits.cpu().numpy().reshape(B, k1, V).astype(np.float64), ref_logits)
+        assert sfv.read_device_status(ws_acc) == 0
+        compare_accept(ref, n.cpu().numpy(), toks.cpu().numpy(), ratio.cpu().numpy())
