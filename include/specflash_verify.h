@@ -37,9 +37,12 @@
  *     so each may start while the previous kernel on `stream` drains.  Before
  *     waiting for that kernel, sf_verify_attention reads the block table, the
  *     sequence lengths and the prefix part of the KV cache (positions below
- *     seq_lens[b] - n_q); these, and the workspace, must not be written by
- *     the kernel immediately before it on the stream.  Everything else (q,
- *     the draft rows' K/V, logits, probabilities, tokens, uniforms) may be.
+ *     seq_lens[b] - n_q), and the LM-head projections read the weights;
+ *     these, and the workspace, must already be in place when the previous
+ *     kernel on the stream starts (so neither it nor a kernel it may overlap
+ *     writes them).  Everything else (q, hidden states, the draft rows' K/V,
+ *     logits, probabilities, tokens, uniforms, temperatures) may come from
+ *     the previous kernel: every kernel waits for it before reading them.
  */
 #ifndef SPECFLASH_VERIFY_H
 #define SPECFLASH_VERIFY_H
@@ -218,7 +221,7 @@ int sf_accept(const float *target_logits, const float *draft_probs,
 /* [8, 2^20].  workspace >= sf_verify_lm_head_accept_workspace_size(B, k, V)*/
 /* bytes, 256-byte aligned, zero-filled before first use.                   */
 /* The weight copies start before the previous kernel on the stream        */
-/* completes (the weights must not be written by it).                       */
+/* completes (the weights must be in place when that kernel starts).        */
 /* ------------------------------------------------------------------------ */
 size_t sf_verify_lm_head_accept_workspace_size(int B, int k, int V);
 
@@ -308,8 +311,8 @@ int sf_kv_commit(int32_t *seq_lens, int32_t *block_table, int32_t *free_pages,
 /* workspace    >= sf_draft_tail_workspace_size(R, V) bytes, 256-byte        */
 /*              aligned, zero-filled before first use (status word).        */
 /* Stream order: the projection copies weight tiles before waiting for the   */
-/* previous kernel on the stream (the weights must not be written by it);    */
-/* hidden, temperature, uniforms and the outputs follow it.                  */
+/* previous kernel on the stream (the weights must be in place when that     */
+/* kernel starts); hidden, temperature, uniforms and the outputs follow it.  */
 /* Results are deterministic; SF_DEVICE_TIMEOUT is the only device status.   */
 /* ------------------------------------------------------------------------ */
 size_t sf_draft_tail_workspace_size(int R, int V);
