@@ -72,7 +72,7 @@ typedef enum {
 #define SF_DEVICE_BAD_SEQLEN 0x8u /* seq_lens[b] outside [n_q, max_pages*16]   */
 #define SF_DEVICE_OUT_OF_PAGES 0x10u /* sf_kv_commit: free-page stack too small */
 
-/* Limits of this build. */
+/* Compile-time limits of the library (calls beyond them return an error). */
 #define SF_PAGE_SIZE 16      /* tokens per KV page                            */
 #define SF_MAX_BATCH 1024    /* sequences per call                            */
 #define SF_MAX_QUERY_ROWS 16 /* n_q: draft rows scored per sequence           */
