@@ -723,9 +723,12 @@ def run_ours(args):
                 "host_result_matches_device": h_ok},
         "launch": "cuda_graph" if use_graph else "eager",
         "eager_ms_per_step": eager_ms,
-        # per step: each layer's attention kernel (+ the merge kernel after the
-        # tcgen05 kernel), then the two acceptance kernels
-        "gpu_launches": args.steps * (L * (2 if kernel == "verify_attention_tc_kernel" else 1) + 2),
+        # per step: each layer's attention launches, then the acceptance's, as
+        # the library reports them for these shapes on this device
+        "gpu_launches": args.steps * (
+            L * sfv.verify_attention_kernel_launches(wl.B, wl.rows, wl.H_q, wl.H_kv, wl.d,
+                                                     att.block_table.shape[2])
+            + sfv.accept_kernel_launches(wl.B, wl.k, wl.V)),
         "clocks": clk,
         "device_status": status,
     }

@@ -990,6 +990,15 @@ size_t sf_accept_workspace_size(int B, int k, int V) {
   return sf::acc_layout(B, k, plan).total;
 }
 
+int sf_accept_kernel_launches(int B, int k, int V) {
+  using namespace sf;
+  if (check_accept_shapes(B, k, V) != SF_OK) return 0;
+  int cs = 0, slice = 0;
+  bool cluster_ok = false;
+  if (cluster_plan(V, &cs, &slice) && cluster_setup(cs, &cluster_ok) != SF_OK) return 0;
+  return cluster_ok ? 1 : 2;
+}
+
 int sf_accept(const float *target_logits, const float *draft_probs,
               const int32_t *draft_tokens, const float *uniforms, const float *temperature,
               int B, int k, int V, int32_t *num_accepted, int32_t *out_tokens,

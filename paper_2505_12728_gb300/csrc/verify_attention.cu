@@ -1077,6 +1077,16 @@ size_t sf_verify_attention_workspace_size(int B, int n_q, int H_q, int H_kv, int
   return sf::attn_layout(B, H_kv, n_q * (H_q / H_kv), head_dim, plan.G).total;
 }
 
+int sf_verify_attention_kernel_launches(int B, int n_q, int H_q, int H_kv, int head_dim,
+                                        int max_pages_per_seq, int page_size, int num_splits) {
+  if (sf::check_shapes(B, n_q, H_q, H_kv, head_dim, page_size, max_pages_per_seq) != SF_OK)
+    return 0;
+  sf::AttnPlan plan;
+  if (sf::plan_attention(B, n_q, H_q, H_kv, head_dim, max_pages_per_seq, num_splits, &plan) != SF_OK)
+    return 0;
+  return plan.tc ? 2 : 1;  // the tcgen05 kernel leaves its merge to verify_merge_kernel
+}
+
 int sf_verify_attention(const void *q, const void *k_cache, const void *v_cache,
                         const int32_t *block_table, const int32_t *seq_lens, int B, int n_q,
                         int H_q, int H_kv, int head_dim, int page_size, int num_pages,

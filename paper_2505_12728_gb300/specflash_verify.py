@@ -28,8 +28,8 @@ PAGE_SIZE = 16
 EXPORTED_SYMBOLS = (
     "sf_status_string", "sf_last_error", "sf_version", "sf_workspace_init",
     "sf_read_device_status", "sf_verify_attention_workspace_size", "sf_verify_attention",
-    "sf_verify_attention_noalloc",
-    "sf_accept_workspace_size", "sf_accept",
+    "sf_verify_attention_noalloc", "sf_verify_attention_kernel_launches",
+    "sf_accept_workspace_size", "sf_accept", "sf_accept_kernel_launches",
     "sf_kv_commit_workspace_size", "sf_kv_commit",
     "sf_draft_tail_workspace_size", "sf_lm_head", "sf_sample", "sf_draft_sample",
     "sf_visual_compress_workspace_size", "sf_visual_compress",
@@ -82,8 +82,12 @@ def load_library(path: str | None = None):
         lib.sf_verify_attention_noalloc.argtypes = [P, P, P, P, P, I, I, I, I, I, I, I, I, F, I,
                                                     P, P, P]
         lib.sf_verify_attention_noalloc.restype = I
+        lib.sf_verify_attention_kernel_launches.argtypes = [I] * 8
+        lib.sf_verify_attention_kernel_launches.restype = I
         lib.sf_accept_workspace_size.argtypes = [I, I, I]
         lib.sf_accept_workspace_size.restype = S
+        lib.sf_accept_kernel_launches.argtypes = [I, I, I]
+        lib.sf_accept_kernel_launches.restype = I
         lib.sf_accept.argtypes = [P, P, P, P, P, I, I, I, P, P, P, P, S, P]
         lib.sf_accept.restype = I
         lib.sf_kv_commit_workspace_size.argtypes = []
@@ -154,6 +158,24 @@ def verify_attention_workspace_size(B, n_q, H_q, H_kv, head_dim, max_pages_per_s
 
 def accept_workspace_size(B, k, V) -> int:
     n = load_library().sf_accept_workspace_size(B, k, V)
+    if n == 0:
+        raise SFError(1, "invalid acceptance shape: " + load_library().sf_last_error().decode())
+    return int(n)
+
+
+def verify_attention_kernel_launches(B, n_q, H_q, H_kv, head_dim, max_pages_per_seq,
+                                     num_splits=0) -> int:
+    """Kernels one verify_attention call with these shapes launches (1 or 2)."""
+    n = load_library().sf_verify_attention_kernel_launches(B, n_q, H_q, H_kv, head_dim,
+                                                           max_pages_per_seq, PAGE_SIZE, num_splits)
+    if n == 0:
+        raise SFError(1, "invalid attention shape: " + load_library().sf_last_error().decode())
+    return int(n)
+
+
+def accept_kernel_launches(B, k, V) -> int:
+    """Kernels one accept call with these shapes launches (1 or 2)."""
+    n = load_library().sf_accept_kernel_launches(B, k, V)
     if n == 0:
         raise SFError(1, "invalid acceptance shape: " + load_library().sf_last_error().decode())
     return int(n)

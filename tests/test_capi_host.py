@@ -71,3 +71,14 @@ def test_invalid_accept_arguments_are_rejected_on_the_host(lib):
     assert call(2, 4, 1) == 1
     assert call(2, 4, 100, ws=None) == 4
     assert lib.sf_accept_workspace_size(2, 0, 100) == 0
+
+
+def test_launch_counts_reject_invalid_shapes_before_touching_a_device():
+    # shapes the calls would reject give 0 without any CUDA call
+    lib = sfv.load_library()
+    assert lib.sf_accept_kernel_launches(0, 5, 32000) == 0
+    assert lib.sf_accept_kernel_launches(1, 17, 32000) == 0
+    assert lib.sf_accept_kernel_launches(1, 5, 1) == 0
+    assert lib.sf_verify_attention_kernel_launches(0, 5, 32, 32, 128, 189, 16, 0) == 0
+    assert lib.sf_verify_attention_kernel_launches(1, 5, 32, 32, 96, 189, 16, 0) == 0
+    assert lib.sf_verify_attention_kernel_launches(1, 5, 32, 32, 128, 189, 32, 0) == 0

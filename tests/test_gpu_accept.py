@@ -191,3 +191,12 @@ def test_repeated_calls_are_bit_identical():
     for x, y in zip(a, b):
         np.testing.assert_array_equal(x, y)
     assert sfv.read_device_status(ws) == 0
+
+
+def test_kernel_launch_counts_follow_the_vocabulary():
+    # one cluster kernel while a row fits 16 slices of 2048 tokens, else the
+    # statistics and draw kernels
+    assert sfv.accept_kernel_launches(1, 5, 32000) == 1
+    assert sfv.accept_kernel_launches(4, 8, 32768) == 1
+    assert sfv.accept_kernel_launches(4, 8, 32769) == 2
+    assert sfv.accept_kernel_launches(8, 6, 152064) == 2
