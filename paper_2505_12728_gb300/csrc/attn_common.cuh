@@ -38,6 +38,18 @@ struct AttnParams {
   int slot_stride;    // floats per partial slot: R*D (O) + R (max) + R (sum), padded to 4
 };
 
+// The softmax weights (x, y) as two bf16 pairs: hi = their bf16 rounding,
+// lo = the bf16 rounding of the remainder, so that hi + lo carries ~16
+// significant bits.  P V is accumulated from both: with P rounded once to
+// bf16 (8 bits) against a row sum l of the unrounded fp32 weights, rows with
+// a handful of visible keys reached an output error of 1.05e-2.
+__device__ __forceinline__ void split_bf16x2(float x, float y, uint32_t &hi, uint32_t &lo) {
+  const __nv_bfloat162 h = __floats2bfloat162_rn(x, y);
+  const __nv_bfloat162 l = __floats2bfloat162_rn(x - __low2float(h), y - __high2float(h));
+  hi = *reinterpret_cast<const uint32_t *>(&h);
+  lo = *reinterpret_cast<const uint32_t *>(&l);
+}
+
 // Floats per partial slot; a multiple of 4 so every slot starts 16-byte aligned.
 __host__ __device__ inline int partial_slot_floats(int R, int D) {
   return (R * (D + 2) + 3) / 4 * 4;

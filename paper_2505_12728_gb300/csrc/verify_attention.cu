@@ -409,21 +409,46 @@ verify_attention_kernel(const __grid_constant__ CUtensorMap tmap_k,
           o[dt][2] *= a1;
           o[dt][3] *= a1;
         }
-        // O += P V
+        // O += P V.  On a sequence's first tile P = P_hi + P_lo, two bf16
+        // terms (split_bf16x2), so that P carries ~16 bits like the fp32 row
+        // sum l: rows with a handful of visible keys, and weight concentrated
+        // on the first keys, otherwise show P's bf16 rounding in the output.
+        // Later tiles use P_hi alone (their weights are spread over many keys).
+        if (lt == 0) {
 #pragma unroll
-        for (int kt = 0; kt < KW / 16; ++kt) {
-          uint32_t pa[4];
-          pa[0] = pack_bf16x2(s[2 * kt][0], s[2 * kt][1]);
-          pa[1] = pack_bf16x2(s[2 * kt][2], s[2 * kt][3]);
-          pa[2] = pack_bf16x2(s[2 * kt + 1][0], s[2 * kt + 1][1]);
-          pa[3] = pack_bf16x2(s[2 * kt + 1][2], s[2 * kt + 1][3]);
-          const int key = ks * KW + kt * 16 + (lane & 7) + ((lane >> 3) & 1) * 8;
+          for (int kt = 0; kt < KW / 16; ++kt) {
+            uint32_t pa[4], pl[4];
+            split_bf16x2(s[2 * kt][0], s[2 * kt][1], pa[0], pl[0]);
+            split_bf16x2(s[2 * kt][2], s[2 * kt][3], pa[1], pl[1]);
+            split_bf16x2(s[2 * kt + 1][0], s[2 * kt + 1][1], pa[2], pl[2]);
+            split_bf16x2(s[2 * kt + 1][2], s[2 * kt + 1][3], pa[3], pl[3]);
+            const int key = ks * KW + kt * 16 + (lane & 7) + ((lane >> 3) & 1) * 8;
 #pragma unroll
-          for (int dt = 0; dt < DT; dt += 2) {
-            uint32_t b0, b1, b2, b3;
-            ldmatrix_x4_trans(vbase + swz<D>(key, dt + (lane >> 4)), b0, b1, b2, b3);
-            mma_bf16_16816(o[dt], pa, b0, b1);
-            mma_bf16_16816(o[dt + 1], pa, b2, b3);
+            for (int dt = 0; dt < DT; dt += 2) {
+              uint32_t b0, b1, b2, b3;
+              ldmatrix_x4_trans(vbase + swz<D>(key, dt + (lane >> 4)), b0, b1, b2, b3);
+              mma_bf16_16816(o[dt], pa, b0, b1);
+              mma_bf16_16816(o[dt], pl, b0, b1);
+              mma_bf16_16816(o[dt + 1], pa, b2, b3);
+              mma_bf16_16816(o[dt + 1], pl, b2, b3);
+            }
+          }
+        } else {
+#pragma unroll
+          for (int kt = 0; kt < KW / 16; ++kt) {
+            uint32_t pa[4];
+            pa[0] = pack_bf16x2(s[2 * kt][0], s[2 * kt][1]);
+            pa[1] = pack_bf16x2(s[2 * kt][2], s[2 * kt][3]);
+            pa[2] = pack_bf16x2(s[2 * kt + 1][0], s[2 * kt + 1][1]);
+            pa[3] = pack_bf16x2(s[2 * kt + 1][2], s[2 * kt + 1][3]);
+            const int key = ks * KW + kt * 16 + (lane & 7) + ((lane >> 3) & 1) * 8;
+#pragma unroll
+            for (int dt = 0; dt < DT; dt += 2) {
+              uint32_t b0, b1, b2, b3;
+              ldmatrix_x4_trans(vbase + swz<D>(key, dt + (lane >> 4)), b0, b1, b2, b3);
+              mma_bf16_16816(o[dt], pa, b0, b1);
+              mma_bf16_16816(o[dt + 1], pa, b2, b3);
+            }
           }
         }
       }

@@ -40,7 +40,11 @@
 //  * One CTA per SM (the ring and Q fill most of shared memory), so the
 //    whole 512-column TMEM is this CTA's: O of the first piece [0,128), O of
 //    later pieces [128,256), S0 [256,320), S1 [320,384), P0 [384,416),
-//    P1 [416,448).
+//    P1 [416,448), and the low bf16 parts of P0 and P1 [448,480), [480,512)
+//    (on a sequence's first tile P V is accumulated from P = P_hi + P_lo, two
+//    bf16 terms, so that it carries P to ~16 bits like the fp32 row sum it
+//    is divided by: rows with a handful of visible keys, and weight
+//    concentrated on the first keys, otherwise show P's bf16 rounding).
 //  * A piece that covers a whole segment writes bf16 out and the LSE; a
 //    split segment's pieces write fp32 partials to the workspace, which the
 //    merge kernel of verify_attention.cu combines.
@@ -64,7 +68,7 @@ constexpr int kTcProducerWarp = 5;
 constexpr uint32_t kTmemCols = 512;
 // O of a CTA's first piece stays in [0,128) until the end (it may be split);
 // every later piece accumulates in [128,256).
-constexpr uint32_t kTmemOFirst = 0, kTmemOLater = 128, kTmemS = 256, kTmemP = 384;
+constexpr uint32_t kTmemOFirst = 0, kTmemOLater = 128, kTmemS = 256, kTmemP = 384, kTmemPlo = 448;
 constexpr float kRescaleLog2 = 8.f;
 constexpr int kTilesBeforeQ = 5;  // K/V tiles copied before the first Q is loaded
 // The segment-aligned partition is used while its largest piece is at most
@@ -308,6 +312,7 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
     uint32_t pv_piece_start = 0;  // first tile of the piece of tile pv
     uint32_t pv_piece_end = 0;
     int pv_piece = -1;            // piece of tile pv
+    int pv_lt0 = 0;               // its first tile within the sequence
     uint32_t t_qk = t_begin, t_pv = t_begin;  // piece cursors (global tiles)
     int q_piece = -1, q_ready = -1;           // piece of tile qk, pieces with Q
     uint32_t total = 0;
@@ -331,6 +336,7 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
         const Piece pc = piece_at(t_pv);
         t_pv += pc.n_tiles;
         pv_piece_start = pv_piece_end;
+        pv_lt0 = pc.lt0;
         ++pv_piece;
         pv_piece_end += pc.n_tiles;
       }
@@ -369,15 +375,17 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
           const uint32_t slot = pv % STAGES;
           const uint32_t vb = ring + slot * L::kStageBytes + L::kTileBytes;
           const bool first = pv == pv_piece_start;
+          const bool seq_first = first && pv_lt0 == 0;  // the sequence's first tile: P_hi + P_lo
           if (elect_one()) {
 #pragma unroll
             for (int j = 0; j < kTileTokens / 16; ++j) {
               // V page j = keys 16j..16j+15 (K): 8-key groups 1024 B apart;
               // the 64-column halves of N are kPageHalfBytes apart
               const uint64_t b = smem_desc_sw128(vb + j * kPageBytes, kPageHalfBytes, 1024);
-              tc_mma_ts(tmem + (pv_piece == 0 ? kTmemOFirst : kTmemOLater),
-                        tmem + kTmemP + (pv & 1u) * 32u + j * 8u, b, kIdescPV,
+              const uint32_t acc = tmem + (pv_piece == 0 ? kTmemOFirst : kTmemOLater);
+              tc_mma_ts(acc, tmem + kTmemP + (pv & 1u) * 32u + j * 8u, b, kIdescPV,
                         (first && j == 0) ? 0u : 1u);
+              if (seq_first) tc_mma_ts(acc, tmem + kTmemPlo + (pv & 1u) * 32u + j * 8u, b, kIdescPV, 1u);
             }
             tc_commit(bar(ODONE + (pv & 1u)));
             tc_commit(bar(EMPTY + slot));
@@ -549,19 +557,22 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
         }
         const float mu = ref == -INFINITY ? 0.f : ref;
         float rs = 0.f;
-        uint32_t mine[KPL / 2];
+        uint32_t mine[KPL / 2], mine_lo[KPL / 2];
 #pragma unroll
         for (int c2 = 0; c2 < KPL / 2; ++c2) {
           const float p0 = fast_exp2(fmaf(x[2 * c2], p.scale_log2, -mu));
           const float p1 = fast_exp2(fmaf(x[2 * c2 + 1], p.scale_log2, -mu));
           rs += p0 + p1;
-          mine[c2] = pack_bf16x2(p0, p1);
+          split_bf16x2(p0, p1, mine[c2], mine_lo[c2]);
         }
         l_run = l_run * alpha + rs;
         // P row of this lane: its keys' weights, zeros for the other lanes' keys
-        uint32_t pk[32];
+        uint32_t pk[32], pk_lo[32];
 #pragma unroll
-        for (int cc = 0; cc < 32; ++cc) pk[cc] = (cc / (KPL / 2) == kap) ? mine[cc % (KPL / 2)] : 0u;
+        for (int cc = 0; cc < 32; ++cc) {
+          pk[cc] = (cc / (KPL / 2) == kap) ? mine[cc % (KPL / 2)] : 0u;
+          pk_lo[cc] = (cc / (KPL / 2) == kap) ? mine_lo[cc % (KPL / 2)] : 0u;
+        }
         // P buffer n&1 is free once the P V of tile n-2 has completed
         if (n >= 2 && !wwait(bar(ODONE + (n & 1u)), ((n - 2) >> 1) & 1u)) {
           ok = false;
@@ -585,6 +596,7 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
           }
         }
         tmem_st_32x32b_x32(tl + kTmemP + (n & 1u) * 32u, pk);
+        if (pc.lt0 + it == 0) tmem_st_32x32b_x32(tl + kTmemPlo + (n & 1u) * 32u, pk_lo);
         tmem_wait_st();
         tc_fence_before_sync();
         mbar_arrive(bar(PFULL + (n & 1u)));

@@ -200,3 +200,14 @@ def test_kernel_launch_counts_follow_the_vocabulary():
     assert sfv.accept_kernel_launches(4, 8, 32768) == 1
     assert sfv.accept_kernel_launches(4, 8, 32769) == 2
     assert sfv.accept_kernel_launches(8, 6, 152064) == 2
+
+
+@pytest.mark.parametrize("V", [32000, 152064])
+@pytest.mark.parametrize("mode", ["sampling", "alternate"])
+def test_longest_draft_matches_oracle(oracle_mod, V, mode):
+    # k = 16 drafts (the limit) on both acceptance paths
+    inp = make_accept_case(8, 16, V, seed=[16, V], mode=mode)
+    ref = oracle_accept(oracle_mod, inp)
+    n, toks, ratio = run_accept(inp)
+    excluded = compare_accept(ref, n, toks, ratio)
+    assert excluded <= 1

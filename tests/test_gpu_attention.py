@@ -244,3 +244,18 @@ def test_kernel_launch_counts_follow_the_rows_per_kv_head():
     assert sfv.verify_attention_kernel_launches(2, 16, 8, 8, 64, 40) == 1
     assert sfv.verify_attention_kernel_launches(4, 8, 28, 4, 128, 305) == 2
     assert sfv.verify_attention_kernel_launches(16, 8, 28, 4, 128, 2049) == 2
+
+
+@pytest.mark.parametrize("n_q,H_q,H_kv,d", [
+    (4, 8, 8, 64),      # mma.sync kernel: 8192 segments of one or two tiles
+    (8, 28, 4, 128),    # tcgen05 kernel: 56 rows per KV head, 4096 segments
+])
+def test_largest_batch_matches_oracle(oracle_mod, n_q, H_q, H_kv, d):
+    # B = 1024 sequences (the batch limit) with ragged prefixes of 0..120
+    # tokens: the on-device tile partition spans every sequence
+    rng = np.random.default_rng(1024 + n_q)
+    prefixes = [int(x) for x in rng.integers(0, 121, size=1024)]
+    case = make_attention_case(1024, n_q, H_q, H_kv, d, prefixes, seed=77 + d)
+    ref_out, ref_lse = oracle_attention(oracle_mod, case)
+    out, lse = run_attention(case, num_splits=0)
+    assert_attention_close(out, lse, ref_out, ref_lse)
