@@ -132,6 +132,11 @@ int sf_read_device_status(const void *workspace, uint32_t *status_out);
 /* lse          fp32 [B][n_q][H_q] (natural log, scaled scores); may be NULL.*/
 /* workspace    >= sf_verify_attention_workspace_size(...) bytes, 256-byte   */
 /*              aligned, zero-filled before first use.                       */
+/* Accuracy: scores and softmax statistics in fp32; P V on bf16 tensor cores */
+/* with P carried as two bf16 terms on each sequence's first 64-token tile   */
+/* and as one on later tiles.  Against the exact result, out is within 1e-2  */
+/* (bf16 rounding of out included, for |out| < 4) and lse within 1e-3 on the */
+/* tested inputs (N(0,1) q, k, v in bf16, 1 to 32K keys).                    */
 /* ------------------------------------------------------------------------ */
 size_t sf_verify_attention_workspace_size(int B, int n_q, int H_q, int H_kv, int head_dim,
                                           int max_pages_per_seq, int page_size,
