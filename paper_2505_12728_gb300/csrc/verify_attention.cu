@@ -22,6 +22,8 @@
 //    the M dimension of bf16 m16n8k16 tensor-core MMAs (S = Q K^T and
 //    O += P V, fp32 accumulate); scores stay in registers, where an fp32
 //    online softmax (base 2, scale folded in) rescales the running output.
+//    On a sequence's first tile P enters P V as two bf16 terms (see
+//    split_bf16x2), so that rows with few visible keys keep P's precision.
 //    The four warps split each tile's keys and combine in shared memory at
 //    the end of a piece.  More rows per KV head (GQA) are a real dense
 //    contraction and go to the tcgen05 kernel in verify_attention_tc.cu.
@@ -36,9 +38,10 @@
 //      - the tcgen05 kernel's split segments (many rows): verify_merge_kernel,
 //        one thread per output quad.
 //  * Launches use programmatic stream serialisation: the partition, the
-//    block-table reads and the first copies of prefix tiles run before
-//    griddepcontrol.wait, overlapping the previous kernel on the stream
-//    (tiles holding draft positions are copied after it).
+//    block-table reads (for one sequence, its whole row copied to shared
+//    memory next to the seq_lens read) and the first copies of prefix tiles
+//    run before griddepcontrol.wait, overlapping the previous kernel on the
+//    stream (tiles holding draft positions are copied after it).
 //  * Page indices outside the pool and positions past a sequence's end are
 //    loaded as zero boxes (TMA out-of-bounds fill); bad indices set a bit in
 //    the status word.  Every mbarrier wait is bounded.
