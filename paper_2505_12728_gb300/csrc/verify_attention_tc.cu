@@ -512,6 +512,7 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
         uint32_t sv[64];
         tmem_ld_32x32b_x64(tl + kTmemS + (n & 1u) * 64u, sv);
         const int tile_pos = (pc.lt0 + it) * kTileTokens;
+        const bool split_p = pc.lt0 + it == 0;  // P as two bf16 terms on the sequence's first tile
         const int valid_keys = pc.T - tile_pos;
         if (valid_keys < kTileTokens) {
           // V rows past the sequence end hold whatever the page holds: zero
@@ -563,16 +564,14 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
           const float p0 = fast_exp2(fmaf(x[2 * c2], p.scale_log2, -mu));
           const float p1 = fast_exp2(fmaf(x[2 * c2 + 1], p.scale_log2, -mu));
           rs += p0 + p1;
-          split_bf16x2(p0, p1, mine[c2], mine_lo[c2]);
+          if (split_p) split_bf16x2(p0, p1, mine[c2], mine_lo[c2]);
+          else mine[c2] = pack_bf16x2(p0, p1);
         }
         l_run = l_run * alpha + rs;
         // P row of this lane: its keys' weights, zeros for the other lanes' keys
-        uint32_t pk[32], pk_lo[32];
+        uint32_t pk[32];
 #pragma unroll
-        for (int cc = 0; cc < 32; ++cc) {
-          pk[cc] = (cc / (KPL / 2) == kap) ? mine[cc % (KPL / 2)] : 0u;
-          pk_lo[cc] = (cc / (KPL / 2) == kap) ? mine_lo[cc % (KPL / 2)] : 0u;
-        }
+        for (int cc = 0; cc < 32; ++cc) pk[cc] = (cc / (KPL / 2) == kap) ? mine[cc % (KPL / 2)] : 0u;
         // P buffer n&1 is free once the P V of tile n-2 has completed
         if (n >= 2 && !wwait(bar(ODONE + (n & 1u)), ((n - 2) >> 1) & 1u)) {
           ok = false;
@@ -596,7 +595,12 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
           }
         }
         tmem_st_32x32b_x32(tl + kTmemP + (n & 1u) * 32u, pk);
-        if (pc.lt0 + it == 0) tmem_st_32x32b_x32(tl + kTmemPlo + (n & 1u) * 32u, pk_lo);
+        if (split_p) {  // the sequence's first tile: P_lo too (warp-uniform)
+          uint32_t pk_lo[32];
+#pragma unroll
+          for (int cc = 0; cc < 32; ++cc) pk_lo[cc] = (cc / (KPL / 2) == kap) ? mine_lo[cc % (KPL / 2)] : 0u;
+          tmem_st_32x32b_x32(tl + kTmemPlo + (n & 1u) * 32u, pk_lo);
+        }
         tmem_wait_st();
         tc_fence_before_sync();
         mbar_arrive(bar(PFULL + (n & 1u)));
