@@ -130,6 +130,12 @@ def _stream_handle(stream):
     return ctypes.c_void_p(s.cuda_stream)
 
 
+def _need_workspace(workspace):
+    """A caller-supplied workspace must be a contiguous uint8 CUDA tensor (its
+    numel() is the byte count passed to the library)."""
+    _need(workspace, "workspace", torch.uint8)
+
+
 def _need(t, name, dtype, shape=None):
     if not isinstance(t, torch.Tensor):
         raise TypeError(f"{name} must be a torch.Tensor")
@@ -187,11 +193,13 @@ def new_workspace(nbytes: int, device=None) -> torch.Tensor:
 
 
 def workspace_init(workspace: torch.Tensor, stream=None):
+    _need_workspace(workspace)
     _check(load_library().sf_workspace_init(_ptr(workspace), workspace.numel(),
                                             _stream_handle(stream)))
 
 
 def read_device_status(workspace: torch.Tensor) -> int:
+    _need_workspace(workspace)
     v = ctypes.c_uint32(0)
     _check(load_library().sf_read_device_status(_ptr(workspace), ctypes.byref(v)))
     return int(v.value)
@@ -209,6 +217,8 @@ def verify_attention(q, k_cache, v_cache, block_table, seq_lens, *, out=None, ls
     or None)."""
     B, n_q, H_q, d = q.shape
     num_pages, H_kv, page, d2 = k_cache.shape
+    if block_table.dim() != 2 or block_table.shape[0] != B:
+        raise ValueError(f"block_table has shape {tuple(block_table.shape)}, expected ({B}, max_pages)")
     _need(q, "q", torch.bfloat16)
     _need(k_cache, "k_cache", torch.bfloat16)
     _need(v_cache, "v_cache", torch.bfloat16, k_cache.shape)
@@ -227,6 +237,7 @@ def verify_attention(q, k_cache, v_cache, block_table, seq_lens, *, out=None, ls
     if workspace is None:
         workspace = new_workspace(verify_attention_workspace_size(
             B, n_q, H_q, H_kv, d, max_pages, page, num_splits), q.device)
+    _need_workspace(workspace)
     _check(load_library().sf_verify_attention(
         _ptr(q), _ptr(k_cache), _ptr(v_cache), _ptr(block_table), _ptr(seq_lens), B, n_q, H_q,
         H_kv, d, page, num_pages, max_pages, float(softmax_scale), int(num_splits), _ptr(out),
@@ -243,6 +254,8 @@ def verify_attention_noalloc(q, k_cache, v_cache, block_table, seq_lens, *, out=
     not supplied."""
     B, n_q, H_q, d = q.shape
     num_pages, H_kv, page, _ = k_cache.shape
+    if block_table.dim() != 2 or block_table.shape[0] != B:
+        raise ValueError(f"block_table has shape {tuple(block_table.shape)}, expected ({B}, max_pages)")
     _need(q, "q", torch.bfloat16)
     _need(k_cache, "k_cache", torch.bfloat16)
     _need(v_cache, "v_cache", torch.bfloat16, k_cache.shape)
@@ -292,6 +305,7 @@ def accept(target_logits, draft_probs, draft_tokens, uniforms, temperature, *,
         _need(accept_ratio, "accept_ratio", torch.float32, (B, k))
     if workspace is None:
         workspace = new_workspace(accept_workspace_size(B, k, V), dev)
+    _need_workspace(workspace)
     _check(load_library().sf_accept(
         _ptr(target_logits), _ptr(draft_probs), _ptr(draft_tokens), _ptr(uniforms),
         _ptr(temperature), B, k, V, _ptr(num_accepted), _ptr(out_tokens), _ptr(accept_ratio),
@@ -338,6 +352,7 @@ def verify_lm_head_accept(hidden, weight, draft_probs, draft_tokens, uniforms, t
         _need(accept_ratio, "accept_ratio", torch.float32, (B, k))
     if workspace is None:
         workspace = new_workspace(verify_lm_head_accept_workspace_size(B, k, V), dev)
+    _need_workspace(workspace)
     _check(load_library().sf_verify_lm_head_accept(
         _ptr(hidden), _ptr(weight), _ptr(draft_probs), _ptr(draft_tokens), _ptr(uniforms),
         _ptr(temperature), B, k, V, d, _ptr(logits), _ptr(num_accepted), _ptr(out_tokens),
@@ -364,6 +379,7 @@ def kv_commit(seq_lens, block_table, free_pages, free_count, num_accepted, n_q, 
     _need(num_accepted, "num_accepted", torch.int32, (B,))
     if workspace is None:
         workspace = new_workspace(kv_commit_workspace_size(), seq_lens.device)
+    _need_workspace(workspace)
     _check(load_library().sf_kv_commit(
         _ptr(seq_lens), _ptr(block_table), _ptr(free_pages), _ptr(free_count), _ptr(num_accepted),
         B, n_q, n_q_next, max_pages, PAGE_SIZE, free_pages.numel(), _ptr(workspace),
@@ -392,6 +408,7 @@ def lm_head(hidden, weight, *, logits=None, workspace=None, stream=None):
     _need(logits, "logits", torch.float32, (R, V))
     if workspace is None:
         workspace = new_workspace(draft_tail_workspace_size(R, V), hidden.device)
+    _need_workspace(workspace)
     _check(load_library().sf_lm_head(_ptr(hidden), _ptr(weight), R, Hd, V, _ptr(logits),
                                      _ptr(workspace), workspace.numel(), _stream_handle(stream)))
     return logits
@@ -414,6 +431,7 @@ def sample(logits, uniforms, temperature, *, probs=None, tokens=None, workspace=
     _need(tokens, "tokens", torch.int32, (R,))
     if workspace is None:
         workspace = new_workspace(draft_tail_workspace_size(R, V), dev)
+    _need_workspace(workspace)
     _check(load_library().sf_sample(_ptr(logits), _ptr(uniforms), _ptr(temperature), R, V,
                                     _ptr(probs), _ptr(tokens), _ptr(workspace), workspace.numel(),
                                     _stream_handle(stream)))
@@ -443,6 +461,7 @@ def draft_sample(hidden, weight, uniforms, temperature, *, logits=None, probs=No
     _need(tokens, "tokens", torch.int32, (R,))
     if workspace is None:
         workspace = new_workspace(draft_tail_workspace_size(R, V), dev)
+    _need_workspace(workspace)
     _check(load_library().sf_draft_sample(
         _ptr(hidden), _ptr(weight), _ptr(uniforms), _ptr(temperature), R, Hd, V, _ptr(logits),
         _ptr(probs), _ptr(tokens), _ptr(workspace), workspace.numel(), _stream_handle(stream)))
@@ -473,6 +492,7 @@ def visual_compress(queries, features, *, out=None, workspace=None, stream=None)
     _need(out, "out", torch.bfloat16, (F, C, d))
     if workspace is None:
         workspace = new_workspace(visual_compress_workspace_size(F, N, C, d), queries.device)
+    _need_workspace(workspace)
     _check(load_library().sf_visual_compress(_ptr(queries), _ptr(features), F, N, C, d, _ptr(out),
                                              _ptr(workspace), workspace.numel(),
                                              _stream_handle(stream)))

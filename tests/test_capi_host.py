@@ -82,3 +82,25 @@ def test_launch_counts_reject_invalid_shapes_before_touching_a_device():
     assert lib.sf_verify_attention_kernel_launches(0, 5, 32, 32, 128, 189, 16, 0) == 0
     assert lib.sf_verify_attention_kernel_launches(1, 5, 32, 32, 96, 189, 16, 0) == 0
     assert lib.sf_verify_attention_kernel_launches(1, 5, 32, 32, 128, 189, 32, 0) == 0
+
+
+def test_binding_rejects_host_tensors_and_bad_shapes_before_any_launch():
+    # the binding checks dtype, device, contiguity and shapes before calling
+    # the library; these run without a GPU because every check fails first
+    import torch
+    bf = torch.zeros((1, 4, 8, 64), dtype=torch.bfloat16)            # host tensor
+    kc = torch.zeros((8, 8, 16, 64), dtype=torch.bfloat16)
+    bt = torch.zeros((1, 8), dtype=torch.int32)
+    sl = torch.full((1,), 20, dtype=torch.int32)
+    with pytest.raises(ValueError, match="CUDA"):
+        sfv.verify_attention(bf, kc, kc, bt, sl)
+    with pytest.raises(TypeError, match="bfloat16"):
+        sfv.verify_attention(bf.float(), kc, kc, bt, sl)
+    with pytest.raises(ValueError, match="block_table"):
+        sfv.verify_attention(bf, kc, kc, torch.zeros((2, 8), dtype=torch.int32), sl)
+    with pytest.raises(ValueError, match="block_table"):
+        sfv.verify_attention(bf, kc, kc, torch.zeros(8, dtype=torch.int32), sl)
+    with pytest.raises(ValueError, match="CUDA"):
+        sfv.read_device_status(torch.zeros(256, dtype=torch.uint8))
+    with pytest.raises(TypeError, match="uint8"):
+        sfv.workspace_init(torch.zeros(64, dtype=torch.int32))
