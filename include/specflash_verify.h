@@ -152,7 +152,8 @@ int sf_verify_attention(const void *q, const void *k_cache, const void *v_cache,
 /* Kernels one sf_verify_attention call with these shapes launches on the    */
 /* current device: 1 (at most 16 rows per KV head: the split kernel merges  */
 /* in place) or 2 (the tcgen05 split kernel, then the merge kernel); 0 for   */
-/* shapes sf_verify_attention rejects.  For graph and launch planning.       */
+/* shapes sf_verify_attention rejects or without a usable CUDA device       */
+/* (sf_last_error says which).  For graph and launch planning.              */
 int sf_verify_attention_kernel_launches(int B, int n_q, int H_q, int H_kv, int head_dim,
                                         int max_pages_per_seq, int page_size, int num_splits);
 
@@ -213,7 +214,8 @@ size_t sf_accept_workspace_size(int B, int k, int V);
 /* Kernels one sf_accept call with these shapes launches on the current      */
 /* device: 1 (a row fits one 16-CTA thread-block cluster, V <= 32768, and    */
 /* such a cluster can be resident) or 2 (statistics, then draw); 0 for       */
-/* shapes sf_accept rejects.  For graph and launch planning.                 */
+/* shapes sf_accept rejects or without a usable CUDA device (sf_last_error  */
+/* says which).  For graph and launch planning.                             */
 int sf_accept_kernel_launches(int B, int k, int V);
 
 int sf_accept(const float *target_logits, const float *draft_probs,
