@@ -175,7 +175,7 @@ def verify_attention_kernel_launches(B, n_q, H_q, H_kv, head_dim, max_pages_per_
     n = load_library().sf_verify_attention_kernel_launches(B, n_q, H_q, H_kv, head_dim,
                                                            max_pages_per_seq, PAGE_SIZE, num_splits)
     if n == 0:
-        raise SFError(1, "invalid attention shape: " + load_library().sf_last_error().decode())
+        raise SFError(1, "no attention launch plan: " + load_library().sf_last_error().decode())
     return int(n)
 
 
@@ -183,7 +183,7 @@ def accept_kernel_launches(B, k, V) -> int:
     """Kernels one accept call with these shapes launches (1 or 2)."""
     n = load_library().sf_accept_kernel_launches(B, k, V)
     if n == 0:
-        raise SFError(1, "invalid acceptance shape: " + load_library().sf_last_error().decode())
+        raise SFError(1, "no acceptance launch plan: " + load_library().sf_last_error().decode())
     return int(n)
 
 
