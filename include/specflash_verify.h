@@ -174,6 +174,10 @@ int sf_verify_attention_kernel_launches(int B, int n_q, int H_q, int H_kv, int h
 /* cudaMemsetAsync on `stream`, then launches the kernel.                    */
 /* Its first call on a device looks up the scratch's device address (once    */
 /* per device, cached); make that first call before any stream capture.      */
+/* The cached address lives as long as the process: resetting a device       */
+/* (cudaDeviceReset) after this entry point has used it is not supported.    */
+/* Every argument check runs before the scratch is touched: a rejected call  */
+/* enqueues nothing.                                                          */
 /* All calls share the one scratch array, which keeps the previous call's    */
 /* contents: calls that may overlap on the GPU (different streams, or        */
 /* threads without ordering) race and give wrong results; serialise them.    */

@@ -881,6 +881,28 @@ static int check_shapes(int B, int n_q, int H_q, int H_kv, int D, int page_size,
   return SF_OK;
 }
 
+// Every argument check of a call that does not need the launch plan: shapes,
+// required pointers, alignment, pool size and scale.
+static int check_call_args(const void *q, const void *k_cache, const void *v_cache,
+                           const int32_t *block_table, const int32_t *seq_lens, int B, int n_q,
+                           int H_q, int H_kv, int head_dim, int page_size, int num_pages,
+                           int max_pages_per_seq, float softmax_scale, const void *out,
+                           const float *lse) {
+  int st = check_shapes(B, n_q, H_q, H_kv, head_dim, page_size, max_pages_per_seq);
+  if (st != SF_OK) return st;
+  if (!q || !k_cache || !v_cache || !block_table || !seq_lens || !out)
+    return fail(SF_ERR_INVALID_ARG, "a required pointer is NULL");
+  if (num_pages < 1) return fail(SF_ERR_INVALID_ARG, "num_pages=%d", num_pages);
+  if ((long long)num_pages * H_kv * SF_PAGE_SIZE >= (1LL << 31))
+    return fail(SF_ERR_UNSUPPORTED, "KV pool of %d pages x %d heads too large", num_pages, H_kv);
+  if (!aligned(q, 16) || !aligned(k_cache, 16) || !aligned(v_cache, 16) || !aligned(out, 16) ||
+      !aligned(block_table, 4) || !aligned(seq_lens, 4) || (lse && !aligned(lse, 4)))
+    return fail(SF_ERR_INVALID_ARG, "q, caches and out must be 16-byte aligned");
+  if (!(softmax_scale >= 0.f) || std::isinf(softmax_scale))
+    return fail(SF_ERR_INVALID_ARG, "softmax_scale must be finite and >= 0");
+  return SF_OK;
+}
+
 struct AttnPlan {
   AttnVariant v;
   int G;
@@ -1123,18 +1145,10 @@ int sf_verify_attention(const void *q, const void *k_cache, const void *v_cache,
                         cudaStream_t stream) {
   using namespace sf;
   clear_error();
-  int st = check_shapes(B, n_q, H_q, H_kv, head_dim, page_size, max_pages_per_seq);
+  int st = check_call_args(q, k_cache, v_cache, block_table, seq_lens, B, n_q, H_q, H_kv,
+                           head_dim, page_size, num_pages, max_pages_per_seq, softmax_scale, out,
+                           lse);
   if (st != SF_OK) return st;
-  if (!q || !k_cache || !v_cache || !block_table || !seq_lens || !out)
-    return fail(SF_ERR_INVALID_ARG, "a required pointer is NULL");
-  if (num_pages < 1) return fail(SF_ERR_INVALID_ARG, "num_pages=%d", num_pages);
-  if ((long long)num_pages * H_kv * SF_PAGE_SIZE >= (1LL << 31))
-    return fail(SF_ERR_UNSUPPORTED, "KV pool of %d pages x %d heads too large", num_pages, H_kv);
-  if (!aligned(q, 16) || !aligned(k_cache, 16) || !aligned(v_cache, 16) || !aligned(out, 16) ||
-      !aligned(block_table, 4) || !aligned(seq_lens, 4) || (lse && !aligned(lse, 4)))
-    return fail(SF_ERR_INVALID_ARG, "q, caches and out must be 16-byte aligned");
-  if (!(softmax_scale >= 0.f) || std::isinf(softmax_scale))
-    return fail(SF_ERR_INVALID_ARG, "softmax_scale must be finite and >= 0");
   if (!workspace || !aligned(workspace, 256))
     return fail(SF_ERR_WORKSPACE, "workspace must be non-NULL and 256-byte aligned");
 
@@ -1248,7 +1262,10 @@ static __device__ __align__(256) uint8_t g_static_scratch[kStaticScratchBytes];
 // Device address of g_static_scratch on the current device.  Host code must
 // not use the symbol itself (it is a host-side stand-in, not a device
 // address); the address is looked up once per device, with that device
-// current, and cached.
+// current, and cached for the life of the process.  A device reset
+// (cudaDeviceReset) destroys the module that holds the array, so the cached
+// address must not outlive it: resetting a device that this entry point has
+// used is not supported.
 static int static_scratch_address(void **out) {
   static std::mutex mu;
   static void *addr[64] = {nullptr};
@@ -1279,7 +1296,11 @@ extern "C" int sf_verify_attention_noalloc(const void *q, const void *k_cache,
                                            cudaStream_t stream) {
   using namespace sf;
   clear_error();
-  int st = check_shapes(B, n_q, H_q, H_kv, head_dim, page_size, max_pages_per_seq);
+  // every argument check first: a rejected call enqueues nothing, not even
+  // the clearing of the shared scratch (another stream may be using it)
+  int st = check_call_args(q, k_cache, v_cache, block_table, seq_lens, B, n_q, H_q, H_kv,
+                           head_dim, page_size, num_pages, max_pages_per_seq, softmax_scale, out,
+                           lse);
   if (st != SF_OK) return st;
   AttnPlan plan;
   st = plan_attention(B, n_q, H_q, H_kv, head_dim, max_pages_per_seq, num_splits, &plan);

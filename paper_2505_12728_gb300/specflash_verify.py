@@ -219,13 +219,13 @@ def verify_attention(q, k_cache, v_cache, block_table, seq_lens, *, out=None, ls
     num_pages, H_kv, page, d2 = k_cache.shape
     if block_table.dim() != 2 or block_table.shape[0] != B:
         raise ValueError(f"block_table has shape {tuple(block_table.shape)}, expected ({B}, max_pages)")
+    if d2 != d:
+        raise ValueError("head_dim of q and caches differ")
     _need(q, "q", torch.bfloat16)
     _need(k_cache, "k_cache", torch.bfloat16)
     _need(v_cache, "v_cache", torch.bfloat16, k_cache.shape)
     _need(block_table, "block_table", torch.int32)
     _need(seq_lens, "seq_lens", torch.int32, (B,))
-    if d2 != d:
-        raise ValueError("head_dim of q and caches differ")
     max_pages = block_table.shape[1]
     if out is None:
         out = torch.empty_like(q)
@@ -253,9 +253,13 @@ def verify_attention_noalloc(q, k_cache, v_cache, block_table, seq_lens, *, out=
     overlap on the GPU race on it).  Outputs may still be allocated here when
     not supplied."""
     B, n_q, H_q, d = q.shape
-    num_pages, H_kv, page, _ = k_cache.shape
+    num_pages, H_kv, page, d2 = k_cache.shape
     if block_table.dim() != 2 or block_table.shape[0] != B:
         raise ValueError(f"block_table has shape {tuple(block_table.shape)}, expected ({B}, max_pages)")
+    if d2 != d:
+        # the library sizes the caches' tensor maps from q's head_dim: a
+        # narrower cache would let the copies read past its end
+        raise ValueError("head_dim of q and caches differ")
     _need(q, "q", torch.bfloat16)
     _need(k_cache, "k_cache", torch.bfloat16)
     _need(v_cache, "v_cache", torch.bfloat16, k_cache.shape)

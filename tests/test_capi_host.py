@@ -104,3 +104,21 @@ def test_binding_rejects_host_tensors_and_bad_shapes_before_any_launch():
         sfv.read_device_status(torch.zeros(256, dtype=torch.uint8))
     with pytest.raises(TypeError, match="uint8"):
         sfv.workspace_init(torch.zeros(64, dtype=torch.int32))
+
+
+def test_binding_rejects_a_cache_narrower_than_q_before_the_library_is_called(monkeypatch):
+    # the library sizes the caches' tensor maps from q's head_dim, so a cache
+    # with a smaller head_dim must be refused by the binding itself
+    import torch
+
+    def no_library():
+        raise AssertionError("the library must not be reached")
+
+    monkeypatch.setattr(sfv, "load_library", no_library)
+    q = torch.zeros((1, 4, 8, 128), dtype=torch.bfloat16)
+    kc = torch.zeros((8, 8, 16, 64), dtype=torch.bfloat16)
+    bt = torch.zeros((1, 8), dtype=torch.int32)
+    sl = torch.full((1,), 20, dtype=torch.int32)
+    for fn in (sfv.verify_attention, sfv.verify_attention_noalloc):
+        with pytest.raises(ValueError, match="head_dim"):
+            fn(q, kc, kc, bt, sl)
