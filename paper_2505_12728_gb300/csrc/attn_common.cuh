@@ -198,7 +198,7 @@ __device__ __forceinline__ T merge_load(const T *p) {
 // The pieces are read in batches of kMergeBatch with an online rescale; all
 // loads of a batch are issued before any is used, so a batch costs one
 // memory round trip.  Partial slot layout: O [R][D], m [R], l [R].
-template <int D, bool kBypassL1>
+template <int D, bool kBypassL1, int BATCH = kMergeBatch>
 __device__ __forceinline__ void merge_one(const float *part0, size_t stride, int R, int r, int c4,
                                           int n_pieces, float4 &o, float &M, float &Ls) {
   const float *mrow = part0 + (size_t)R * D + r;
@@ -208,11 +208,11 @@ __device__ __forceinline__ void merge_one(const float *part0, size_t stride, int
   M = -INFINITY;
   Ls = 0.f;
   float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-  for (int q0 = 0; q0 < n_pieces; q0 += kMergeBatch) {
-    float mv[kMergeBatch], lv[kMergeBatch];
-    float4 xv[kMergeBatch];
+  for (int q0 = 0; q0 < n_pieces; q0 += BATCH) {
+    float mv[BATCH], lv[BATCH];
+    float4 xv[BATCH];
 #pragma unroll
-    for (int u = 0; u < kMergeBatch; ++u) {
+    for (int u = 0; u < BATCH; ++u) {
       const bool in = q0 + u < n_pieces;
       mv[u] = in ? merge_load<kBypassL1>(mrow + (q0 + u) * stride) : -INFINITY;
       lv[u] = in ? merge_load<kBypassL1>(lrow + (q0 + u) * stride) : 0.f;
@@ -220,12 +220,12 @@ __device__ __forceinline__ void merge_one(const float *part0, size_t stride, int
     }
     float Mb = M;
 #pragma unroll
-    for (int u = 0; u < kMergeBatch; ++u) Mb = fmaxf(Mb, mv[u]);
+    for (int u = 0; u < BATCH; ++u) Mb = fmaxf(Mb, mv[u]);
     const float a = exp2f(M - Mb);  // first batch: M = -inf, a = 0
     Ls *= a;
     acc.x *= a; acc.y *= a; acc.z *= a; acc.w *= a;
 #pragma unroll
-    for (int u = 0; u < kMergeBatch; ++u) {
+    for (int u = 0; u < BATCH; ++u) {
       const float w = exp2f(mv[u] - Mb);
       Ls += lv[u] * w;
       acc.x += xv[u].x * w; acc.y += xv[u].y * w; acc.z += xv[u].z * w; acc.w += xv[u].w * w;
@@ -237,8 +237,9 @@ __device__ __forceinline__ void merge_one(const float *part0, size_t stride, int
 }
 
 // Host side of the tcgen05 kernel (verify_attention_tc.cu).
-// Dynamic shared memory of a launch for batch B (0 if head_dim is not built).
-int tc_smem_bytes(int head_dim, int B);
+// Dynamic shared memory of a launch with R rows per KV head and batch B (0
+// if head_dim is not built).
+int tc_smem_bytes(int head_dim, int R, int B);
 // Raises the kernel's shared-memory limit once per device.
 int tc_setup(int head_dim, int device);
 // Launches the tcgen05 split kernel over G CTAs.

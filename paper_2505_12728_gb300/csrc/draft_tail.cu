@@ -190,14 +190,24 @@ lm_head_kernel(const __grid_constant__ CUtensorMap tmap_w, const __grid_constant
     s_misc[2] = 0;
     s_misc[3] = 0;
   }
-  if (warp == kLmMmaWarp) {
-    tmem_alloc(smem_addr(s_misc), p.tmem_cols);
-    tmem_relinquish_alloc_permit();
-    tc_fence_before_sync();
+  __syncthreads();  // barrier initialisation visible to every role
+  // Tensor memory is allocated only once the previous kernel on the stream
+  // has completed: a predecessor that is still waiting for its own
+  // predecessor may not have allocated yet, and holding TMEM here while it
+  // waits for columns could deadlock the pair.  The producer warp does not
+  // need TMEM and starts its weight copies meanwhile.
+  uint32_t tmem = 0;
+  if (warp != kLmProducerWarp) {
+    if (warp == kLmMmaWarp) {
+      grid_dependency_wait();
+      tmem_alloc(smem_addr(s_misc), p.tmem_cols);
+      tmem_relinquish_alloc_permit();
+      tc_fence_before_sync();
+    }
+    named_bar_sync(3, kLmEpiThreads + 32);
+    tc_fence_after_sync();
+    tmem = static_cast<uint32_t>(s_misc[0]);
   }
-  __syncthreads();
-  tc_fence_after_sync();
-  const uint32_t tmem = static_cast<uint32_t>(s_misc[0]);
 
   if (warp == kLmProducerWarp) {
     if (lane == 0) {

@@ -775,44 +775,50 @@ verify_attention_kernel(const __grid_constant__ CUtensorMap tmap_k,
 }
 
 // Merge for shapes with many rows per KV head (GQA): the pieces of every
-// split segment are combined by a grid with one thread per 4 output columns
-// of a row (the whole output at once), in piece order (deterministic):
+// split segment are combined by a grid-stride loop with one item per 4
+// output columns of a row, in piece order (deterministic):
 //   M = max_q m_q,  L = sum_q l_q 2^(m_q - M),  O = sum_q 2^(m_q - M) O_q / L,
 //   lse = (M + log2 L) ln 2.
-// Pieces are read in batches of kMergeBatch with a running (online) rescale,
-// so a batch costs one memory round trip.  Launched right after the split
-// kernel with programmatic stream serialisation: its CTAs may be scheduled
-// while the split grid drains, and wait for it before reading anything.
+// Pieces are read in batches of kMergeBatchGqa with a running (online)
+// rescale, so a batch costs one memory round trip.  Launched right after the
+// split kernel with programmatic stream serialisation: its CTAs are
+// scheduled while the split grid runs and wait for it before reading
+// anything.  At most 64 registers per thread, so that several of its CTAs
+// fit next to a split CTA and the whole grid is resident (and has let the
+// next kernel be scheduled) before the split grid completes.
 constexpr int kMergeThreads = 128;
+constexpr int kMergeBatchGqa = 8;
 
 template <int D>
-__global__ void __launch_bounds__(kMergeThreads)
+__global__ void __launch_bounds__(kMergeThreads, 8)
 verify_merge_kernel(const __grid_constant__ AttnParams p) {
   constexpr float kLn2 = 0.6931471805599453f;
-  constexpr int C4 = D / 4;                       // threads per row
+  constexpr int C4 = D / 4;                       // items per row
   grid_launch_dependents();
   grid_dependency_wait();
-  const long long item = (long long)blockIdx.x * kMergeThreads + threadIdx.x;
   const int per_seg = p.R * C4;
-  if (item >= (long long)per_seg * p.B * p.H_kv) return;
-  const int seg = static_cast<int>(item / per_seg);
-  const int rem = static_cast<int>(item % per_seg);
-  const int r = rem / C4, c4 = rem % C4;
-  const int2 desc = p.seg_desc[seg];              // {first CTA, pieces}
-  if (desc.y <= 1) return;                        // the split kernel wrote it
+  const long long total = (long long)per_seg * p.B * p.H_kv;
   const size_t stride = (size_t)p.slot_stride;
-  float4 ov;
-  float M, Ls;
-  merge_one<D, false>(p.partials + (size_t)(desc.x + seg) * stride, stride, p.R, r, c4, desc.y,
-                      ov, M, Ls);
-  const int b = seg / p.H_kv, h_kv = seg % p.H_kv;
-  const int i = r / p.group, j = r % p.group;
-  const size_t row = ((size_t)b * p.n_q + i) * p.H_q + (size_t)h_kv * p.group + j;
-  uint2 packed;
-  packed.x = pack_bf16x2(ov.x, ov.y);
-  packed.y = pack_bf16x2(ov.z, ov.w);
-  *reinterpret_cast<uint2 *>(p.out + row * D + 4 * c4) = packed;
-  if (p.lse && c4 == 0) p.lse[row] = (M + log2f(Ls)) * kLn2;
+  for (long long item = (long long)blockIdx.x * kMergeThreads + threadIdx.x; item < total;
+       item += (long long)gridDim.x * kMergeThreads) {
+    const int seg = static_cast<int>(item / per_seg);
+    const int rem = static_cast<int>(item % per_seg);
+    const int r = rem / C4, c4 = rem % C4;
+    const int2 desc = p.seg_desc[seg];            // {first CTA, pieces}
+    if (desc.y <= 1) continue;                    // the split kernel wrote it
+    float4 ov;
+    float M, Ls;
+    merge_one<D, false, kMergeBatchGqa>(p.partials + (size_t)(desc.x + seg) * stride, stride, p.R,
+                                        r, c4, desc.y, ov, M, Ls);
+    const int b = seg / p.H_kv, h_kv = seg % p.H_kv;
+    const int i = r / p.group, j = r % p.group;
+    const size_t row = ((size_t)b * p.n_q + i) * p.H_q + (size_t)h_kv * p.group + j;
+    uint2 packed;
+    packed.x = pack_bf16x2(ov.x, ov.y);
+    packed.y = pack_bf16x2(ov.z, ov.w);
+    *reinterpret_cast<uint2 *>(p.out + row * D + 4 * c4) = packed;
+    if (p.lse && c4 == 0) p.lse[row] = (M + log2f(Ls)) * kLn2;
+  }
 }
 
 // --------------------------------------------------------------------------
@@ -1008,10 +1014,10 @@ static int plan_attention(int B, int n_q, int H_q, int H_kv, int D, int max_page
     // tensor cores with one CTA per SM (the whole TMEM is one CTA's).
     plan->tc = 1;
     plan->cs = 1;
-    plan->smem = tc_smem_bytes(D, B);
-    if (tc_smem_bytes(D, SF_MAX_BATCH) > dev.max_smem_optin)
+    plan->smem = tc_smem_bytes(D, R, B);
+    if (tc_smem_bytes(D, R, SF_MAX_BATCH) > dev.max_smem_optin)
       return fail(SF_ERR_UNSUPPORTED, "needs %d B shared memory, device allows %d",
-                  tc_smem_bytes(D, SF_MAX_BATCH), dev.max_smem_optin);
+                  tc_smem_bytes(D, R, SF_MAX_BATCH), dev.max_smem_optin);
     st = tc_setup(D, dev.ordinal);
     if (st != SF_OK) return st;
     long long G = num_splits > 0 && num_splits < dev.sm_count ? num_splits : dev.sm_count;
@@ -1075,30 +1081,38 @@ static int plan_attention(int B, int n_q, int H_q, int H_kv, int D, int max_page
 }
 
 // TMA descriptors of the K and V caches, cached by (address, rows,
-// head_dim, box) so that repeated calls on the same caches skip the encoding.
-// half_boxes = 0: one box brings a whole page (both 64-column halves when
-// head_dim is 128); 1: one box brings one 64-column half of a page.
+// head_dim, layout) so that repeated calls on the same caches skip the
+// encoding.  Each box brings one 16-token page; layout 0 lands it as
+// [64-column half][16 tokens][128 B], layout 1 (head_dim 128 only) as
+// [8-token group][half][8 tokens][128 B], so that the 8-token atoms of one
+// half sit at a fixed 2048-byte stride across the pages of a tile.
 static int cache_tensor_map(CUtensorMap *out, const void *base, uint64_t rows, int head_dim,
-                            int half_boxes) {
+                            int layout) {
   static std::mutex mu;
   static std::map<std::tuple<const void *, uint64_t, int, int>, CUtensorMap> maps;
+  if (head_dim != 128) layout = 0;
   {
     std::lock_guard<std::mutex> lock(mu);
-    auto it = maps.find({base, rows, head_dim, half_boxes});
+    auto it = maps.find({base, rows, head_dim, layout});
     if (it != maps.end()) {
       *out = it->second;
       return SF_OK;
     }
   }
-  // head_dim 128: view each 256-byte token row as two 128-byte halves with
-  // the halves outermost, {64 elements, rows, 2 halves} with byte strides
-  // {256, 128}, so a {64, 16, 2} box brings a whole page in the shared
-  // layout [half][token][64] and a {64, 16, 1} box one half of a page.
-  // head_dim 64: {64, rows}, box {64, 16}.
+  // head_dim 128, layout 0: view each 256-byte token row as two 128-byte
+  // halves with the halves outermost, {64 elements, rows, 2 halves} with byte
+  // strides {256, 128}; a {64, 16, 2} box brings a page as [half][token][64].
+  // Layout 1: {64 elements, 8 tokens, 2 halves, rows / 8 token groups} with
+  // byte strides {256, 128, 2048}; a {64, 8, 2, 2} box brings a page as
+  // [group][half][token][64].  head_dim 64: {64, rows}, box {64, 16}.
   int st;
-  if (head_dim == 128) {
+  if (head_dim == 128 && layout == 1) {
+    const uint64_t dims[4] = {64, 8, 2, rows / 8}, strides[3] = {256, 128, 2048};
+    const uint32_t box[4] = {64, 8, 2, 2};
+    st = encode_tensor_map_bf16(out, base, 4, dims, strides, box);
+  } else if (head_dim == 128) {
     const uint64_t dims[3] = {64, rows, 2}, strides[2] = {256, 128};
-    const uint32_t box[3] = {64, SF_PAGE_SIZE, half_boxes ? 1u : 2u};
+    const uint32_t box[3] = {64, SF_PAGE_SIZE, 2};
     st = encode_tensor_map_bf16(out, base, 3, dims, strides, box);
   } else {
     const uint64_t dims[2] = {64, rows}, strides[1] = {128};
@@ -1108,7 +1122,7 @@ static int cache_tensor_map(CUtensorMap *out, const void *base, uint64_t rows, i
   if (st != SF_OK) return st;
   std::lock_guard<std::mutex> lock(mu);
   if (maps.size() >= 4096) maps.clear();
-  maps.emplace(std::make_tuple(base, rows, head_dim, half_boxes), *out);
+  maps.emplace(std::make_tuple(base, rows, head_dim, layout), *out);
   return SF_OK;
 }
 
@@ -1162,7 +1176,7 @@ int sf_verify_attention(const void *q, const void *k_cache, const void *v_cache,
 
   const uint64_t rows = (uint64_t)num_pages * H_kv * SF_PAGE_SIZE;
   CUtensorMap tk, tv;
-  st = cache_tensor_map(&tk, k_cache, rows, head_dim, plan.tc);
+  st = cache_tensor_map(&tk, k_cache, rows, head_dim, plan.tc ? 1 : 0);
   if (st != SF_OK) return st;
   st = cache_tensor_map(&tv, v_cache, rows, head_dim, 0);
   if (st != SF_OK) return st;

@@ -6,51 +6,60 @@
 // computes (Sec. 3.1: the K draft tokens are scored in one forward pass, so
 // each of the n_q new rows attends to the prefix plus the causal draft
 // block), with the same fp32 partial format, so verify_merge_kernel combines
-// split segments.  What differs:
+// split segments.  Design points:
+//  * One CTA per SM with a six-stage ring (192 KB): the prefix tiles of the
+//    ring are copied before griddepcontrol.wait, so they land while the
+//    previous kernel on the stream finishes.  Tensor memory (all 512
+//    columns) is allocated only after that wait: a kernel that waits for
+//    its predecessor never holds TMEM, so two kernels cannot each hold what
+//    the other waits for.
 //  * The work partition is chosen on the device from seq_lens: the
 //    balanced one (all tiles cut into G equal ranges; a CTA may hold pieces
 //    of several segments) or a segment-aligned one (each segment gets
 //    ceil(tiles / Ta) CTAs and every CTA one piece) when its largest piece
-//    is within kAlignSlackTiles of the balanced share -- a CTA's second
-//    piece costs another Q load, epilogue and pipeline start.
-//  * All R rows of a KV head are the M = 128 side of the MMAs.  Row r sits
-//    in TMEM lane 32 * (r % 4) + r / 4, so the rows spread over the four lane
-//    quarters (one per softmax warp); lanes >= R hold zero rows.
-//  * A K tile sits in shared memory as [64-column half][64 tokens][128 B],
-//    128B-swizzled (one TMA box per page and half), so the 64 keys of a half
-//    are eight 8-row swizzle atoms 1024 bytes apart and S = Q K^T is
-//    head_dim/16 MMAs of M=128, N=64, K=16 straight into TMEM.  A V tile sits
-//    as [page][half][16 tokens][128 B] (one box per page: a box costs the
-//    TMA unit about the same whatever its size, so V takes half as many);
-//    P = exp2(S') goes back to TMEM as bf16, and O += P V is four MMAs (one
-//    per page of 16 keys) with A from TMEM and B = V as an MN-major operand
-//    (N = head_dim, the halves 2 KB apart).
-//  * Warp roles: warps 0-3 own one TMEM lane (= one query row) per thread
-//    and run the online softmax with no shuffles; warp 4 allocates TMEM and
-//    runs the MMA loop (one elected lane issues); warp 5 reads the block
-//    table and issues the TMA copies into a STAGES-deep ring.
-//  * Hand-offs are mbarriers: full / empty per ring slot (TMA bytes, MMA
-//    commit), s_full / p_full / o_done per S and P buffer (two of each, so
-//    Q K^T of tile n+1 runs while tile n is in the softmax), q_full per piece.
+//    is within kAlignSlackTiles of the balanced share.
+//  * All R rows of a KV head are the M = 128 side of the MMAs.  The rows are
+//    repeated F = 128 / RPK times (RPK = 32, 64 or 128 rows per copy): copy
+//    kap occupies TMEM lanes [kap * RPK, (kap + 1) * RPK) and, in the
+//    softmax, owns keys [kap * KPL, (kap + 1) * KPL) of every 64-key tile
+//    (KPL = 64 / F).  A copy is a whole number of 32-lane quarters, so each
+//    softmax warp reads exactly its keys' score columns.  The repeated rows
+//    cost the 128-row MMAs nothing; the F partial states of a row merge
+//    through shared memory at the end of a piece.
+//  * Q lives in tensor memory (the A operand of S = Q K^T): each softmax
+//    thread writes its lane's row.  Four S buffers: P = exp2(S') is written
+//    as bf16 over the scores it came from, so Q K^T of tile n+4 (which
+//    overwrites the buffer) is issued after P V of tile n, and tcgen05 MMAs
+//    of one thread execute in issue order.  The softmax of four tiles can be
+//    in flight behind one another.
+//  * A K tile sits in shared memory as [page][8-token group][64-column
+//    half][8 tokens][128 B], 128B-swizzled: one 4-D TMA box per 16-token
+//    page brings both halves, and the 8-token atoms of a half are 2048 bytes
+//    apart, so S = Q K^T is head_dim/16 MMAs of M=128, N=64, K=16.  A V tile
+//    sits as [page][half][16 tokens][128 B] (one box per page); P =
+//    exp2(S') goes back to its S buffer as bf16 and O += P V is four MMAs
+//    (one per page) with A = P from TMEM and B = V as an MN-major operand.
+//    Eight TMA boxes per 32 KB tile, issued by two producer warps (K and V).
+//  * Warp roles: warps 0-3 softmax and epilogue (one TMEM lane quarter
+//    each), warp 4 allocates TMEM and issues the MMAs (one elected lane),
+//    warp 5 reads the block table and issues the K boxes, warp 6 the V
+//    boxes.
+//  * Hand-offs are mbarriers: full / empty per ring slot, s_full / p_full /
+//    o_done per S buffer, q_full per piece.
 //  * The running maximum is a reference that moves only when a row's new
-//    maximum exceeds it by more than kRescaleLog2 (base-2 units): the
-//    weights exp2(x - ref) stay below 2^kRescaleLog2, and the O rescale (a
-//    TMEM read-modify-write that must wait for the previous P V) is rare.
-//    O/l and the LSE do not depend on the reference.
-//  * One CTA per SM (the ring and Q fill most of shared memory), so the
-//    whole 512-column TMEM is this CTA's: O of the first piece [0,128), O of
-//    later pieces [128,256), S0 [256,320), S1 [320,384), P0 [384,416),
-//    P1 [416,448), and the low bf16 parts of P0 and P1 [448,480), [480,512)
-//    (on a sequence's first tile P V is accumulated from P = P_hi + P_lo, two
-//    bf16 terms, so that it carries P to ~16 bits like the fp32 row sum it
-//    is divided by: rows with a handful of visible keys, and weight
-//    concentrated on the first keys, otherwise show P's bf16 rounding).
+//    maximum exceeds it by more than kRescaleLog2 (base-2 units), so the O
+//    rescale (a TMEM read-modify-write behind the previous P V) is rare.
+//  * On a sequence's first tile P V is accumulated from P = P_hi + P_lo, two
+//    bf16 terms, so that P carries ~16 bits like the fp32 row sum it is
+//    divided by (rows with a handful of visible keys would otherwise show
+//    P's bf16 rounding).
 //  * A piece that covers a whole segment writes bf16 out and the LSE; a
 //    split segment's pieces write fp32 partials to the workspace, which the
 //    merge kernel of verify_attention.cu combines.
-//  * The first copies run before griddepcontrol.wait only for tiles that lie
-//    wholly in the prefix; tiles holding draft positions (which the previous
-//    kernel on the stream may have just written) are copied after it.
+//  * K/V copies run before griddepcontrol.wait only for tiles that lie
+//    wholly in the prefix; tiles holding draft positions
+//    (which the previous kernel on the stream may have just written) are
+//    copied after it, and so is Q.
 //  * Every wait is bounded; a timeout sets SF_DEVICE_TIMEOUT, stops every
 //    role, waits (bounded) for copies and MMAs in flight and frees TMEM.
 #include <cmath>
@@ -61,69 +70,98 @@
 
 namespace sf {
 
-constexpr int kTcThreads = 192;
+constexpr int kTcThreads = 224;
 constexpr int kTcSoftmaxThreads = 128;
 constexpr int kTcMmaWarp = 4;
-constexpr int kTcProducerWarp = 5;
+constexpr int kTcKWarp = 5;
+constexpr int kTcVWarp = 6;
 constexpr uint32_t kTmemCols = 512;
-// O of a CTA's first piece stays in [0,128) until the end (it may be split);
-// every later piece accumulates in [128,256).
-constexpr uint32_t kTmemOFirst = 0, kTmemOLater = 128, kTmemS = 256, kTmemP = 384, kTmemPlo = 448;
+constexpr int kNumS = 4;  // S buffers (64 columns each)
+// TMEM columns: O [0, D), Q [128, 128 + D/2), S_b [192 + 64 b, 256 + 64 b);
+// within S_b the bf16 P of the tile overwrites columns [0, 32) and, on a
+// sequence's first tile, its low part P_lo columns [32, 64).
+constexpr uint32_t kTmemO = 0, kTmemQ = 128, kTmemS = 192;
 constexpr float kRescaleLog2 = 8.f;
-constexpr int kTilesBeforeQ = 5;  // K/V tiles copied before the first Q is loaded
 // The segment-aligned partition is used while its largest piece is at most
 // this many tiles above the balanced share (a second piece in a CTA costs
 // about that much: another Q load, epilogue and pipeline start).
 constexpr int kAlignSlackTiles = 3;
+// Registers per thread: low enough that several merge-kernel CTAs fit next
+// to a split CTA on its SM.
+constexpr int kTcMaxRegs = 168;
+constexpr int kTcNamedTmem = 1;     // softmax warps + MMA warp: TMEM allocated
+constexpr int kTcNamedSoftmax = 2;  // softmax warps: epilogue exchange
 
 template <int D>
 struct TcConfig {
-  static constexpr int kStages = D == 128 ? 5 : 8;
+  static constexpr int kStages = D == 128 ? 6 : 12;  // 192 KB of ring either way
 };
 
-template <int D, int STAGES>
+template <int D, int STAGES, int F>
 struct TcSmem {
   static constexpr int kTileBytes = kTileTokens * D * 2;  // one tensor, one tile
   static constexpr int kStageBytes = 2 * kTileBytes;      // K then V
-  static constexpr int kQOffset = STAGES * kStageBytes;
-  static constexpr int kQBytes = 128 * D * 2;             // [D/64][128 rows][128 B]
-  static constexpr int kBarOffset = kQOffset + kQBytes;
-  // full[S], empty[S], s_full[2], p_full[2], o_done[2], q_full, fin
-  static constexpr int kNumBars = 2 * STAGES + 8;
+  static constexpr int kBarOffset = STAGES * kStageBytes;
+  // full[S], empty[S], s_full[NS], p_full[NS], o_done[NS], q_full, fin
+  static constexpr int kNumBars = 2 * STAGES + 3 * kNumS + 2;
   static constexpr int kMiscOffset = kBarOffset + 8 * kNumBars;
   static constexpr int kMiscInts = 16;
-  static constexpr int kPrefixOffset = kMiscOffset + 4 * kMiscInts;
+  static constexpr int kRowsPerCopy = 128 / F;
+  // epilogue exchange: (max, sum) of every lane, then 32 O columns of the
+  // copies kap > 0, column-major so that a warp's stores hit distinct banks
+  static constexpr int kMlOffset = kMiscOffset + 4 * kMiscInts;  // float2 [128]
+  static constexpr int kXOffset = kMlOffset + 8 * 128;            // float [F-1][32][RPK]
+  static constexpr int kXFloats = (F - 1) * 32 * kRowsPerCopy;
+  static constexpr int kPrefixOffset = kXOffset + 4 * kXFloats;
   // tiles prefix [B+1] | seq lens [B] | aligned CTA prefix [B+1]
   static int bytes(int B) { return 1024 + kPrefixOffset + 4 * (3 * B + 3); }
 };
 
+// tcgen05.ld / st of N consecutive 32-bit columns of the thread's lane.
+template <int N>
+__device__ __forceinline__ void tmem_ld_cols(uint32_t taddr, uint32_t (&v)[N]) {
+  if constexpr (N == 64) tmem_ld_32x32b_x64(taddr, v);
+  else if constexpr (N == 32) tmem_ld_32x32b_x32(taddr, v);
+  else if constexpr (N == 16) tmem_ld_32x32b_x16(taddr, v);
+  else tmem_ld_32x32b_x8(taddr, v);
+}
+template <int N>
+__device__ __forceinline__ void tmem_st_cols(uint32_t taddr, const uint32_t (&v)[N]) {
+  if constexpr (N == 32) tmem_st_32x32b_x32(taddr, v);
+  else if constexpr (N == 16) tmem_st_32x32b_x16(taddr, v);
+  else tmem_st_32x32b_x8(taddr, v);
+}
+
 template <int D, int STAGES, int F>
-__global__ void __launch_bounds__(kTcThreads, 1)
+__global__ void __maxnreg__(kTcMaxRegs)
 verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
                            const __grid_constant__ CUtensorMap tmap_v,
                            const __grid_constant__ AttnParams p) {
-  using L = TcSmem<D, STAGES>;
+  using L = TcSmem<D, STAGES, F>;
   constexpr int HALVES = D / 64;
-  constexpr int kPageHalfBytes = kPageTokens * kRowBytes;       // 16 tokens x 64 columns
-  constexpr int kPageBytes = HALVES * kPageHalfBytes;           // one page of V
-  constexpr int kTileHalfBytes = kTileTokens * kRowBytes;       // 64 tokens x 64 columns
-  constexpr int kQHalfBytes = 128 * kRowBytes;                  // 128 rows x 64 columns of Q
+  constexpr int kPageHalfBytes = kPageTokens * kRowBytes;  // 16 tokens x 64 columns
+  constexpr int kPageBytes = HALVES * kPageHalfBytes;      // one page of one tensor
+  constexpr int RPK = 128 / F;                             // M rows per key copy
+  constexpr int KPL = 64 / F;                              // keys per lane and tile
+  constexpr uint32_t kKSbo = HALVES == 2 ? 2048u : 1024u;  // 8-key atoms of a K tile
   constexpr float kLn2 = 0.6931471805599453f;
-  constexpr uint32_t kIdescQK = idesc_bf16_f32(128, 64, 0, 0);  // Q K-major, K K-major
+  constexpr uint32_t kIdescQK = idesc_bf16_f32(128, 64, 0, 0);  // Q (TMEM), K K-major
   constexpr uint32_t kIdescPV = idesc_bf16_f32(128, D, 0, 1);   // P (TMEM), V MN-major
+  constexpr int kQWords = D / 2;                                 // 32-bit columns of a Q row
   // barrier indices
-  constexpr int FULL = 0, EMPTY = STAGES, SFULL = 2 * STAGES, PFULL = 2 * STAGES + 2,
-                ODONE = 2 * STAGES + 4, QFULL = 2 * STAGES + 6, FIN = 2 * STAGES + 7;
+  constexpr int FULL = 0, EMPTY = STAGES, SFULL = 2 * STAGES, PFULL = SFULL + kNumS,
+                ODONE = PFULL + kNumS, QFULL = ODONE + kNumS, FIN = QFULL + 1;
+  constexpr uint32_t NS = kNumS;
 
   extern __shared__ uint8_t smem_raw[];
   uint8_t *smem = reinterpret_cast<uint8_t *>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
   const uint32_t ring = smem_addr(smem);
-  const uint32_t qs = ring + L::kQOffset;
   const uint32_t bars = ring + L::kBarOffset;
   auto bar = [&](int i) -> uint32_t { return bars + 8u * static_cast<uint32_t>(i); };
   int *s_misc = reinterpret_cast<int *>(smem + L::kMiscOffset);
-  // s_misc: [0] TMEM base, [1] abort word, [2] tiles issued, [3] tiles consumed
+  // s_misc: [0] TMEM base, [1] abort word, [2] tiles with K issued, [3] tiles
+  // whose full barrier the MMA warp observed, [4] tiles with V issued
   volatile int *s_abort = s_misc + 1;
   int *s_prefix = reinterpret_cast<int *>(smem + L::kPrefixOffset);
   int *s_len = s_prefix + p.B + 1;
@@ -134,10 +172,10 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
   grid_launch_dependents();
   if (tid == 0) {
     for (int s = 0; s < STAGES; ++s) {
-      mbar_init(bar(FULL + s), 1);
+      mbar_init(bar(FULL + s), 2);  // one arrival per producer warp (with its bytes)
       mbar_init(bar(EMPTY + s), 1);
     }
-    for (int x = 0; x < 2; ++x) {
+    for (int x = 0; x < kNumS; ++x) {
       mbar_init(bar(SFULL + x), 1);
       mbar_init(bar(PFULL + x), kTcSoftmaxThreads);
       mbar_init(bar(ODONE + x), 1);
@@ -150,6 +188,7 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
     s_misc[1] = 0;
     s_misc[2] = 0;
     s_misc[3] = 0;
+    s_misc[4] = 0;
   }
   tile_prefix<kTcThreads>(p, s_prefix, s_len, s_misc + 8);
   __syncthreads();
@@ -208,43 +247,34 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
     return aligned ? apc : locate_piece(t, t_end, part, s_prefix, s_len, p);
   };
 
-  if (warp == kTcMmaWarp) {
-    tmem_alloc(smem_addr(s_misc), kTmemCols);
-    tmem_relinquish_alloc_permit();
-    tc_fence_before_sync();
-  }
-  __syncthreads();
-  tc_fence_after_sync();
-  const uint32_t tmem = static_cast<uint32_t>(s_misc[0]);
-
-  if (warp == kTcProducerWarp) {
+  if (warp == kTcKWarp || warp == kTcVWarp) {
     // ------------------------------------------------------------------
-    // producer: the warp reads the block table; one lane per TMA box (K:
-    // page and half, V: page) issues the copies of a tile
+    // producers: lanes 0-3 of the K warp issue the K boxes of a tile (one
+    // per page), lanes 0-3 of the V warp its V boxes; each warp arrives on
+    // the slot's full barrier with its own bytes.
     // ------------------------------------------------------------------
+    const bool is_k = warp == kTcKWarp;
     const uint64_t policy = l2_policy_evict_first();
     bool waited = false;
-    bool q_in = false;  // Q of the first piece is in shared memory
-    uint32_t n = 0;     // tiles issued by this CTA
+    uint32_t n = 0;  // tiles issued by this CTA
     bool ok = true;
     for (uint32_t t = t_begin; t < t_end && ok;) {
       const Piece pc = piece_at(t);
       t += pc.n_tiles;
+      // page ids of tiles base .. base+7 of the piece: lane l holds tile
+      // base + l/4, page l%4
+      auto window = [&](int base) -> int {
+        const int lt = pc.lt0 + base + (lane >> 2);
+        const int lp = lt * kPagesPerTile + (lane & 3);
+        int id = kBeyondEnd;
+        if (base + (lane >> 2) < pc.n_tiles && lp * kPageTokens < pc.T)
+          id = p.block_table[(size_t)pc.b * p.max_pages + lp];
+        return id;
+      };
       int ids = kBeyondEnd;
       for (int it = 0; it < pc.n_tiles; ++it, ++n) {
-        if ((it & 7) == 0) {
-          // page ids of tiles it .. it+7: lane l holds tile it + l/4, page l%4
-          const int lt = pc.lt0 + it + (lane >> 2);
-          const int lp = lt * kPagesPerTile + (lane & 3);
-          ids = kBeyondEnd;
-          if (it + (lane >> 2) < pc.n_tiles && lp * kPageTokens < pc.T)
-            ids = p.block_table[(size_t)pc.b * p.max_pages + lp];
-        }
-        // lanes 0 .. 4*HALVES-1 issue the K boxes (page l / HALVES, half
-        // l % HALVES), the next four lanes the V boxes (one per page)
-        constexpr int kKBoxes = HALVES * kPagesPerTile;
-        const bool is_v = lane >= kKBoxes;
-        const int pg = is_v ? (lane - kKBoxes) & (kPagesPerTile - 1) : (lane / HALVES) & (kPagesPerTile - 1);
+        if ((it & 7) == 0) ids = window(it);
+        const int pg = lane & 3;
         const int phys = __shfl_sync(0xffffffffu, ids, ((it & 7) << 2) + pg);
         const int slot = static_cast<int>(n % STAGES);
         if (n >= static_cast<uint32_t>(STAGES)) {
@@ -261,58 +291,55 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
           grid_dependency_wait();
           waited = true;
         }
-        // Q goes first: beyond kTilesBeforeQ tiles, the copies would queue
-        // ahead of the Q loads that the first MMA needs
-        if (!q_in && n >= static_cast<uint32_t>(kTilesBeforeQ)) {
-          int w = 1;
-          if (lane == 0) w = mbar_wait_or_abort(bar(QFULL), 0, s_abort);
-          if (!__shfl_sync(0xffffffffu, w, 0)) {
-            ok = false;
-            break;
-          }
-          q_in = true;
-        }
-        if (lane == 0) mbar_arrive_expect_tx(bar(FULL + slot), L::kStageBytes);
+        if (lane == 0) mbar_arrive_expect_tx(bar(FULL + slot), L::kTileBytes);
         __syncwarp();
-        if (lane < kKBoxes + kPagesPerTile) {
+        if (lane < kPagesPerTile) {
           // pages past the sequence end or outside the pool load as zeros
           int row = p.oob_row;
           if (phys != kBeyondEnd) {
-            if (phys < 0 || phys >= p.num_pages) set_status(p.status, SF_DEVICE_BAD_PAGE);
-            else row = (phys * p.H_kv + pc.h_kv) * kPageTokens;
+            if (phys < 0 || phys >= p.num_pages) {
+              if (is_k) set_status(p.status, SF_DEVICE_BAD_PAGE);
+            } else {
+              row = (phys * p.H_kv + pc.h_kv) * kPageTokens;
+            }
           }
           const uint32_t stage = ring + slot * L::kStageBytes;
-          if (is_v) {
-            // whole page: [half][16 tokens][128 B]
+          if (is_k) {
+            const uint32_t dst = stage + pg * kPageBytes;
+            if constexpr (HALVES == 2) tma_load_4d(dst, &tmap_k, 0, 0, 0, row / 8, bar(FULL + slot), policy);
+            else tma_load_2d(dst, &tmap_k, 0, row, bar(FULL + slot), policy);
+          } else {
             const uint32_t dst = stage + L::kTileBytes + pg * kPageBytes;
             if constexpr (HALVES == 2) tma_load_3d(dst, &tmap_v, 0, row, 0, bar(FULL + slot), policy);
             else tma_load_2d(dst, &tmap_v, 0, row, bar(FULL + slot), policy);
-          } else {
-            const int h = lane % HALVES;
-            const uint32_t dst = stage + h * kTileHalfBytes + pg * kPageHalfBytes;
-            if constexpr (HALVES == 2) tma_load_3d(dst, &tmap_k, 0, row, h, bar(FULL + slot), policy);
-            else tma_load_2d(dst, &tmap_k, 0, row, bar(FULL + slot), policy);
           }
         }
         __syncwarp();
+        if (lane == 0) s_misc[is_k ? 2 : 4] = static_cast<int>(n + 1);
       }
     }
-    if (lane == 0) s_misc[2] = static_cast<int>(n);
   } else if (warp == kTcMmaWarp) {
     // ------------------------------------------------------------------
-    // MMA loop: the whole warp polls, one elected lane issues and commits.
-    // Q K^T of tile m needs its K tile (full), S buffer m&1 read out
-    // (p_full of tile m-2, i.e. m <= pv + 1) and, for the first tile of a
+    // MMA warp.  TMEM is allocated after the previous kernel on the stream
+    // has completed.  Then the whole warp polls, one elected lane issues and
+    // commits.  Q K^T of tile m needs its K tile (full), its S buffer free
+    // (P V of tile m - NS issued: the MMAs run in issue order, so that P V
+    // reads its P before Q K^T overwrites it) and, for the first tile of a
     // piece, the piece's Q (q_full); P V of tile m needs its P (p_full).
-    // The two streams are issued as soon as their conditions hold, so a
-    // P V never waits behind the next tile's copy.
+    // The two streams are issued as soon as their conditions hold.
     // ------------------------------------------------------------------
+    grid_dependency_wait();
+    tmem_alloc(smem_addr(s_misc), kTmemCols);
+    tmem_relinquish_alloc_permit();
+    tc_fence_before_sync();
+    named_bar_sync(kTcNamedTmem, kTcSoftmaxThreads + 32);
+    tc_fence_after_sync();
+    const uint32_t tmem = static_cast<uint32_t>(s_misc[0]);
     uint32_t qk = 0, pv = 0;      // next tile to multiply, CTA-wide counters
     uint32_t qk_piece_end = 0;    // end of the piece of tile qk
     uint32_t pv_piece_start = 0;  // first tile of the piece of tile pv
     uint32_t pv_piece_end = 0;
-    int pv_piece = -1;            // piece of tile pv
-    int pv_lt0 = 0;               // its first tile within the sequence
+    int pv_lt0 = 0;               // first tile of pv's piece within its sequence
     uint32_t t_qk = t_begin, t_pv = t_begin;  // piece cursors (global tiles)
     int q_piece = -1, q_ready = -1;           // piece of tile qk, pieces with Q
     uint32_t total = 0;
@@ -325,7 +352,6 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
     bool ok = true;
     while (pv < total && ok) {
       bool progress = false;
-      // advance the piece cursors
       if (qk == qk_piece_end && qk < total) {
         const Piece pc = piece_at(t_qk);
         t_qk += pc.n_tiles;
@@ -337,10 +363,9 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
         t_pv += pc.n_tiles;
         pv_piece_start = pv_piece_end;
         pv_lt0 = pc.lt0;
-        ++pv_piece;
         pv_piece_end += pc.n_tiles;
       }
-      if (qk < total && qk <= pv + 1) {
+      if (qk < total && qk < pv + NS) {
         bool ready = true;
         if (q_ready < q_piece) {
           ready = mbar_test_wait(bar(QFULL), static_cast<uint32_t>(q_piece) & 1u);
@@ -352,16 +377,15 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
           tc_fence_after_sync();
           if (lane == 0) s_misc[3] = static_cast<int>(qk + 1);
           const uint32_t kb = ring + slot * L::kStageBytes;
-          const uint32_t d = tmem + kTmemS + (qk & 1u) * 64u;
+          const uint32_t d = tmem + kTmemS + (qk % NS) * 64u;
           if (elect_one()) {
 #pragma unroll
             for (int kk = 0; kk < D / 16; ++kk) {
-              const uint32_t koff = (kk >> 2) * kQHalfBytes + (kk & 3) * 32;
-              const uint64_t a = smem_desc_sw128(qs + koff, 16, 1024);
-              const uint64_t b = smem_desc_sw128(kb + (kk >> 2) * kTileHalfBytes + (kk & 3) * 32, 16, 1024);
-              tc_mma_ss(d, a, b, kIdescQK, kk > 0 ? 1u : 0u);
+              // K step kk: columns 16kk .. 16kk+15 = 32-byte column kk%4 of half kk/4
+              const uint64_t b = smem_desc_sw128(kb + (kk >> 2) * 1024 + (kk & 3) * 32, 16, kKSbo);
+              tc_mma_ts(d, tmem + kTmemQ + kk * 8, b, kIdescQK, kk > 0 ? 1u : 0u);
             }
-            tc_commit(bar(SFULL + (qk & 1u)));
+            tc_commit(bar(SFULL + qk % NS));
           }
           __syncwarp();
           ++qk;
@@ -369,7 +393,7 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
         }
       }
       if (pv < qk) {
-        const bool ready = mbar_test_wait(bar(PFULL + (pv & 1u)), (pv >> 1) & 1u);
+        const bool ready = mbar_test_wait(bar(PFULL + pv % NS), (pv / NS) & 1u);
         if (__all_sync(0xffffffffu, ready)) {
           tc_fence_after_sync();
           const uint32_t slot = pv % STAGES;
@@ -382,12 +406,11 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
               // V page j = keys 16j..16j+15 (K): 8-key groups 1024 B apart;
               // the 64-column halves of N are kPageHalfBytes apart
               const uint64_t b = smem_desc_sw128(vb + j * kPageBytes, kPageHalfBytes, 1024);
-              const uint32_t acc = tmem + (pv_piece == 0 ? kTmemOFirst : kTmemOLater);
-              tc_mma_ts(acc, tmem + kTmemP + (pv & 1u) * 32u + j * 8u, b, kIdescPV,
-                        (first && j == 0) ? 0u : 1u);
-              if (seq_first) tc_mma_ts(acc, tmem + kTmemPlo + (pv & 1u) * 32u + j * 8u, b, kIdescPV, 1u);
+              const uint32_t pb = tmem + kTmemS + (pv % NS) * 64u + j * 8u;
+              tc_mma_ts(tmem + kTmemO, pb, b, kIdescPV, (first && j == 0) ? 0u : 1u);
+              if (seq_first) tc_mma_ts(tmem + kTmemO, pb + 32u, b, kIdescPV, 1u);
             }
-            tc_commit(bar(ODONE + (pv & 1u)));
+            tc_commit(bar(ODONE + pv % NS));
             tc_commit(bar(EMPTY + slot));
           }
           __syncwarp();
@@ -414,103 +437,89 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
     (void)mbar_wait_bounded(bar(FIN), 0);
   } else {
     // ------------------------------------------------------------------
-    // softmax + epilogue.  Lane quarter q = warp; inside it, lane
-    // rho + k * (32/F) holds query row r = 4 * rho + q for the k-th 1/F of
-    // the tile's keys (the Q row is repeated F times on the M side, which
-    // costs the 128-row MMAs nothing).  Each lane keeps its own reference,
-    // sum and O over its keys; the F lanes of a row merge at the end of the
-    // piece with shuffles, like split-KV pieces.
+    // softmax + epilogue.  Thread tid owns TMEM lane tid: key copy kap =
+    // tid / RPK (keys kap*KPL .. kap*KPL+KPL-1 of every tile) of query row
+    // r = tid % RPK (rows >= R are padding).  Each lane keeps its own
+    // reference, sum and O over its keys.
     // ------------------------------------------------------------------
-    constexpr int RPQ = 32 / F;    // rows per lane quarter
-    constexpr int KPL = 64 / F;    // keys per lane and tile
-    const int rho = lane % RPQ, kap = lane / RPQ;
-    const int r = rho * 4 + warp;
+    const int kap = tid / RPK, r = tid % RPK;
     const bool valid = r < p.R;
-    const uint32_t tl = tmem + (static_cast<uint32_t>(warp * 32) << 16);
+    const int qi = valid ? r / p.group : 0, qj = valid ? r % p.group : 0;
+    float2 *s_ml = reinterpret_cast<float2 *>(smem + L::kMlOffset);
+    float *s_x = reinterpret_cast<float *>(smem + L::kXOffset);
     // every lane waits (and acquires); the warp leaves together if any failed,
     // so the warp-collective tcgen05 instructions always see a full warp
     auto wwait = [&](uint32_t b, uint32_t parity) -> bool {
       const bool w = mbar_wait_or_abort(b, parity, s_abort);
       return __all_sync(0xffffffffu, w);
     };
-    bool waited = false;
+    auto q_row = [&](const Piece &pc) -> const __nv_bfloat16 * {
+      return p.q + (((size_t)pc.b * p.n_q + qi) * p.H_q + (size_t)pc.h_kv * p.group + qj) * D;
+    };
+    // this lane's Q row of piece pc into TMEM (zeros for padding rows)
+    auto load_q = [&](const Piece &pc, uint32_t tl) {
+      uint32_t qw[kQWords];
+      const uint4 *src = reinterpret_cast<const uint4 *>(q_row(pc));
+#pragma unroll
+      for (int u = 0; u < D / 8; ++u) {
+        const uint4 v = valid ? __ldg(src + u) : make_uint4(0u, 0u, 0u, 0u);
+        qw[4 * u] = v.x; qw[4 * u + 1] = v.y; qw[4 * u + 2] = v.z; qw[4 * u + 3] = v.w;
+      }
+#pragma unroll
+      for (int c = 0; c < kQWords; c += 32) {
+        uint32_t part[32];
+#pragma unroll
+        for (int k = 0; k < 32; ++k) part[k] = qw[c + k];
+        tmem_st_32x32b_x32(tl + kTmemQ + c, part);
+      }
+    };
+
+    Piece pc0{};
+    if (t_begin < t_end) {
+      pc0 = piece_at(t_begin);
+      if (valid) {
+        const char *row = reinterpret_cast<const char *>(q_row(pc0));
+        for (int x = 0; x < D * 2; x += 128) prefetch_l2(row + x);
+      }
+    }
+    grid_dependency_wait();
+    named_bar_sync(kTcNamedTmem, kTcSoftmaxThreads + 32);
+    tc_fence_after_sync();
+    const uint32_t tmem = static_cast<uint32_t>(s_misc[0]);
+    const uint32_t tl = tmem + (static_cast<uint32_t>(warp * 32) << 16);
+    if (t_begin < t_end) load_q(pc0, tl);
+    tmem_wait_st();
+    tc_fence_before_sync();
+    mbar_arrive(bar(QFULL));
+
     uint32_t n = 0;
     bool ok = true;
-    int pi = 0;                          // piece index in this CTA
-    for (uint32_t t = t_begin; t < t_end && ok; ++pi) {
-      const Piece pc = piece_at(t);
+    int pi = 0;  // piece index in this CTA
+    for (uint32_t t = t_begin; t < t_end; ++pi) {
+      const Piece pc = pi == 0 ? pc0 : piece_at(t);
       t += pc.n_tiles;
-      const uint32_t ob = pi == 0 ? kTmemOFirst : kTmemOLater;  // this piece's O
-      if (!waited) {
-        // Q rows into L2 while the previous kernel drains (a prefetch has
-        // no effect on the values read after the wait)
-        for (int x = tid; x < p.R * (D * 2 / 128); x += kTcSoftmaxThreads) {
-          const int rr = x / (D * 2 / 128), half = x % (D * 2 / 128);
-          const int i = rr / p.group, j = rr % p.group;
-          prefetch_l2(p.q + (((size_t)pc.b * p.n_q + i) * p.H_q + (size_t)pc.h_kv * p.group + j) * D + half * 64);
-        }
-        grid_dependency_wait();
-        waited = true;
-      }
       if (pc.lt0 == 0 && tid == 0) p.seg_desc[pc.seg] = make_int2(pc.c_first, pc.n_pieces);
-
-      // Q rows of the piece into shared memory (every MMA of the previous
-      // piece has completed): M-side row m holds query row
-      // 4 * ((m % 32) % RPQ) + m / 32, 128B-swizzled like the K tiles
-      // (each distinct row is loaded once and stored F times; all loads
-      // first, then all stores: one memory round trip)
-      {
-        constexpr int kQChunks = 4 * RPQ * (D / 8) / kTcSoftmaxThreads;
-        uint4 qv[kQChunks];
-#pragma unroll
-        for (int u = 0; u < kQChunks; ++u) {
-          const int idx = tid + u * kTcSoftmaxThreads;
-          const int ui = idx / (D / 8), c = idx % (D / 8);
-          const int rr = (ui % RPQ) * 4 + ui / RPQ;
-          qv[u] = make_uint4(0u, 0u, 0u, 0u);
-          if (rr < p.R) {
-            const int i = rr / p.group, j = rr % p.group;
-            qv[u] = __ldg(reinterpret_cast<const uint4 *>(
-                p.q + (((size_t)pc.b * p.n_q + i) * p.H_q + (size_t)pc.h_kv * p.group + j) * D + c * 8));
-          }
-        }
-#pragma unroll
-        for (int u = 0; u < kQChunks; ++u) {
-          const int idx = tid + u * kTcSoftmaxThreads;
-          const int ui = idx / (D / 8), c = idx % (D / 8);
-#pragma unroll
-          for (int k = 0; k < F; ++k) {
-            const int mrow = (ui / RPQ) * 32 + ui % RPQ + k * RPQ;
-            *reinterpret_cast<uint4 *>(smem + L::kQOffset + (c >> 3) * kQHalfBytes + mrow * kRowBytes +
-                                       (((c & 7) ^ (mrow & 7)) << 4)) = qv[u];
-          }
-        }
-      }
-      fence_proxy_async_smem();
-      tc_fence_before_sync();
-      mbar_arrive(bar(QFULL));
       if (t < t_end) {
-        // the next piece's Q rows into L2 (one 128-byte line per thread)
+        // the next piece's Q rows into L2 (read after this piece's tiles)
         const Piece nx = piece_at(t);
-        const int lines = p.R * (D * 2 / 128);
-        for (int x = tid; x < lines; x += kTcSoftmaxThreads) {
-          const int rr = x / (D * 2 / 128), half = x % (D * 2 / 128);
-          const int i = rr / p.group, j = rr % p.group;
-          prefetch_l2(p.q + (((size_t)nx.b * p.n_q + i) * p.H_q + (size_t)nx.h_kv * p.group + j) * D + half * 64);
+        if (valid) {
+          const char *row = reinterpret_cast<const char *>(q_row(nx));
+          for (int x = 0; x < D * 2; x += 128) prefetch_l2(row + x);
         }
       }
 
       // last visible key position of this row (draft row i sees L_b + i)
-      const int lim = valid ? pc.Lb + min(r / p.group, p.n_q - 1) : -1;
+      const int lim = valid ? pc.Lb + min(qi, p.n_q - 1) : -1;
       float ref = -INFINITY, l_run = 0.f;
-      for (int it = 0; it < pc.n_tiles; ++it, ++n) {
-        if (!wwait(bar(SFULL + (n & 1u)), (n >> 1) & 1u)) {
+      for (int it = 0; it < pc.n_tiles && ok; ++it, ++n) {
+        const uint32_t sb = tl + kTmemS + (n % NS) * 64u;  // this tile's S buffer
+        if (!wwait(bar(SFULL + n % NS), (n / NS) & 1u)) {
           ok = false;
           break;
         }
         tc_fence_after_sync();
-        uint32_t sv[64];
-        tmem_ld_32x32b_x64(tl + kTmemS + (n & 1u) * 64u, sv);
+        uint32_t sv[KPL];
+        tmem_ld_cols<KPL>(sb + kap * KPL, sv);
         const int tile_pos = (pc.lt0 + it) * kTileTokens;
         const bool split_p = pc.lt0 + it == 0;  // P as two bf16 terms on the sequence's first tile
         const int valid_keys = pc.T - tile_pos;
@@ -528,25 +537,17 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
         }
         // this lane's keys kap*KPL .. kap*KPL + KPL-1 (raw scores; the
         // scale, > 0, is applied to the maximum and folded into the exponent)
-        float x[KPL];
         float mx = -INFINITY;
 #pragma unroll
-        for (int c = 0; c < KPL; ++c) {
-          uint32_t v = sv[c];
-#pragma unroll
-          for (int k = 1; k < F; ++k)
-            if (kap == k) v = sv[k * KPL + c];
-          x[c] = __uint_as_float(v);
-          mx = fmaxf(mx, x[c]);
-        }
+        for (int c = 0; c < KPL; ++c) mx = fmaxf(mx, __uint_as_float(sv[c]));
         const int key0 = tile_pos + kap * KPL;
         if (key0 + KPL - 1 > lim) {
           // causal mask of the draft block, positions past the end, padding rows
           mx = -INFINITY;
 #pragma unroll
           for (int c = 0; c < KPL; ++c) {
-            if (key0 + c > lim) x[c] = -INFINITY;
-            mx = fmaxf(mx, x[c]);
+            if (key0 + c > lim) sv[c] = __float_as_uint(-INFINITY);
+            mx = fmaxf(mx, __uint_as_float(sv[c]));
           }
         }
         mx *= p.scale_log2;
@@ -561,26 +562,17 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
         uint32_t mine[KPL / 2], mine_lo[KPL / 2];
 #pragma unroll
         for (int c2 = 0; c2 < KPL / 2; ++c2) {
-          const float p0 = fast_exp2(fmaf(x[2 * c2], p.scale_log2, -mu));
-          const float p1 = fast_exp2(fmaf(x[2 * c2 + 1], p.scale_log2, -mu));
+          const float p0 = fast_exp2(fmaf(__uint_as_float(sv[2 * c2]), p.scale_log2, -mu));
+          const float p1 = fast_exp2(fmaf(__uint_as_float(sv[2 * c2 + 1]), p.scale_log2, -mu));
           rs += p0 + p1;
           if (split_p) split_bf16x2(p0, p1, mine[c2], mine_lo[c2]);
           else mine[c2] = pack_bf16x2(p0, p1);
         }
         l_run = l_run * alpha + rs;
-        // P row of this lane: its keys' weights, zeros for the other lanes' keys
-        uint32_t pk[32];
-#pragma unroll
-        for (int cc = 0; cc < 32; ++cc) pk[cc] = (cc / (KPL / 2) == kap) ? mine[cc % (KPL / 2)] : 0u;
-        // P buffer n&1 is free once the P V of tile n-2 has completed
-        if (n >= 2 && !wwait(bar(ODONE + (n & 1u)), ((n - 2) >> 1) & 1u)) {
-          ok = false;
-          break;
-        }
         if (__any_sync(0xffffffffu, alpha != 1.f)) {
           // O *= alpha after the P V of tile n-1 (it > 0 here: the first
           // tile of a piece starts with ref = -inf, so alpha = 1)
-          if (!wwait(bar(ODONE + ((n - 1) & 1u)), ((n - 1) >> 1) & 1u)) {
+          if (!wwait(bar(ODONE + (n - 1) % NS), ((n - 1) / NS) & 1u)) {
             ok = false;
             break;
           }
@@ -588,60 +580,93 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
 #pragma unroll 1
           for (int ch = 0; ch < D / 32; ++ch) {
             uint32_t ov[32];
-            tmem_ld_32x32b_x32(tl + ob + ch * 32, ov);
+            tmem_ld_32x32b_x32(tl + kTmemO + ch * 32, ov);
 #pragma unroll
             for (int c = 0; c < 32; ++c) ov[c] = __float_as_uint(__uint_as_float(ov[c]) * alpha);
-            tmem_st_32x32b_x32(tl + ob + ch * 32, ov);
+            tmem_st_32x32b_x32(tl + kTmemO + ch * 32, ov);
           }
         }
-        tmem_st_32x32b_x32(tl + kTmemP + (n & 1u) * 32u, pk);
-        if (split_p) {  // the sequence's first tile: P_lo too (warp-uniform)
-          uint32_t pk_lo[32];
+        // P over the scores: this lane's keys, zeros for the other copies'
+        // keys (the A operand of P V covers the whole tile)
+        {
+          uint32_t pk[32];
 #pragma unroll
-          for (int cc = 0; cc < 32; ++cc) pk_lo[cc] = (cc / (KPL / 2) == kap) ? mine_lo[cc % (KPL / 2)] : 0u;
-          tmem_st_32x32b_x32(tl + kTmemPlo + (n & 1u) * 32u, pk_lo);
+          for (int c = 0; c < 32; ++c) pk[c] = (c / (KPL / 2) == kap) ? mine[c % (KPL / 2)] : 0u;
+          tmem_st_32x32b_x32(sb, pk);
+          if (split_p) {  // the sequence's first tile: P_lo too (warp-uniform)
+#pragma unroll
+            for (int c = 0; c < 32; ++c) pk[c] = (c / (KPL / 2) == kap) ? mine_lo[c % (KPL / 2)] : 0u;
+            tmem_st_32x32b_x32(sb + 32, pk);
+          }
         }
         tmem_wait_st();
         tc_fence_before_sync();
-        mbar_arrive(bar(PFULL + (n & 1u)));
+        mbar_arrive(bar(PFULL + n % NS));
       }
-      if (!ok) break;
+
+      // ---- the next piece's Q (every Q K^T of this piece has completed:
+      // its last score tile was read above), so that the next piece's first
+      // Q K^T overlaps this epilogue ----
+      if (ok && t < t_end) {
+        load_q(piece_at(t), tl);
+        tmem_wait_st();
+        tc_fence_before_sync();
+        mbar_arrive(bar(QFULL));
+      }
 
       // ---- epilogue of the piece ----
-      const uint32_t last = n - 1;
-      if (!wwait(bar(ODONE + (last & 1u)), (last >> 1) & 1u)) {
+      if (ok) {
+        const uint32_t last = n - 1;
+        ok = wwait(bar(ODONE + last % NS), (last / NS) & 1u);
+      }
+      // all four warps take the exchange barriers below, or all skip them
+      if (!named_bar_and(kTcNamedSoftmax, kTcSoftmaxThreads, ok)) {
         ok = false;
         break;
       }
       tc_fence_after_sync();
-      // merge the F lanes of each row (M = max ref, w = 2^(ref - M)); a
-      // whole segment is normalised and written, a split one leaves its
-      // fp32 partial O [R][D] (relative to M), M [R], L [R] in the workspace
-      float M = ref;
+      // merge the F copies of each row (M = max reference, w = 2^(ref - M));
+      // copy 0 then normalises and writes a whole segment, or leaves a split
+      // one's fp32 partial O [R][D] (relative to M), M [R], L [R]
+      float M = ref, Ls = l_run;
+      if constexpr (F > 1) {
+        s_ml[tid] = make_float2(ref, l_run);
+        named_bar_sync(kTcNamedSoftmax, kTcSoftmaxThreads);
 #pragma unroll
-      for (int k = RPQ; k < 32; k <<= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, k));
+        for (int k = 0; k < F; ++k) M = fmaxf(M, s_ml[k * RPK + r].x);
+        Ls = 0.f;
+#pragma unroll
+        for (int k = 0; k < F; ++k) {
+          const float2 v = s_ml[k * RPK + r];
+          if (v.x != -INFINITY) Ls += v.y * exp2f(v.x - M);
+        }
+      }
       const float w = ref == -INFINITY ? 0.f : exp2f(ref - M);
-      float Ls = l_run * w;
-#pragma unroll
-      for (int k = RPQ; k < 32; k <<= 1) Ls += __shfl_xor_sync(0xffffffffu, Ls, k);
-      // tcgen05.ld is warp-collective: every lane loads; lane kap == 0 of a
-      // valid row stores
       const bool writer = valid && kap == 0;
-      const int i = valid ? r / p.group : 0, j = valid ? r % p.group : 0;
-      const size_t row = ((size_t)pc.b * p.n_q + i) * p.H_q + (size_t)pc.h_kv * p.group + j;
+      const size_t row = ((size_t)pc.b * p.n_q + qi) * p.H_q + (size_t)pc.h_kv * p.group + qj;
       const bool whole = pc.n_pieces == 1;
       const float inv = whole ? 1.f / Ls : 1.f;
       float *part0 = p.partials + (size_t)(blockIdx.x + pc.seg) * p.slot_stride;
 #pragma unroll 1
       for (int ch = 0; ch < D / 32; ++ch) {
         uint32_t ov[32];
-        tmem_ld_32x32b_x32(tl + ob + ch * 32, ov);
+        tmem_ld_32x32b_x32(tl + kTmemO + ch * 32, ov);
         float o[32];
 #pragma unroll
-        for (int c = 0; c < 32; ++c) {
-          o[c] = __uint_as_float(ov[c]) * w;
+        for (int c = 0; c < 32; ++c) o[c] = __uint_as_float(ov[c]) * w;
+        if constexpr (F > 1) {
+          if (kap > 0) {
 #pragma unroll
-          for (int k = RPQ; k < 32; k <<= 1) o[c] += __shfl_xor_sync(0xffffffffu, o[c], k);
+            for (int c = 0; c < 32; ++c) s_x[((kap - 1) * 32 + c) * RPK + r] = o[c];
+          }
+          named_bar_sync(kTcNamedSoftmax, kTcSoftmaxThreads);
+          if (kap == 0) {
+#pragma unroll
+            for (int k = 1; k < F; ++k) {
+#pragma unroll
+              for (int c = 0; c < 32; ++c) o[c] += s_x[((k - 1) * 32 + c) * RPK + r];
+            }
+          }
         }
         if (writer && whole) {
           uint4 *dst = reinterpret_cast<uint4 *>(p.out + row * D + ch * 32);
@@ -660,6 +685,7 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
           for (int q4 = 0; q4 < 8; ++q4)
             dst[q4] = make_float4(o[4 * q4], o[4 * q4 + 1], o[4 * q4 + 2], o[4 * q4 + 3]);
         }
+        if constexpr (F > 1) named_bar_sync(kTcNamedSoftmax, kTcSoftmaxThreads);
       }
       if (writer) {
         if (whole) {
@@ -670,8 +696,8 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
         }
       }
       tc_fence_before_sync();
+      if (!ok) break;
     }
-
     tc_fence_before_sync();
   }
 
@@ -679,18 +705,24 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
   __syncthreads();
   if (*s_abort) {
     if (tid == 0) set_status(p.status, SF_DEVICE_TIMEOUT);
-    if (warp == kTcProducerWarp && lane == 0) {
-      // copies issued but never consumed: wait (bounded) until they land
-      for (uint32_t x = static_cast<uint32_t>(s_misc[3]); x < static_cast<uint32_t>(s_misc[2]); ++x)
+    if (warp == kTcKWarp && lane == 0) {
+      // copies issued but never consumed: a tile that only one producer warp
+      // reached gets the other warp's arrival here, then every issued copy
+      // is waited for (bounded) before the shared memory is released
+      const uint32_t kI = static_cast<uint32_t>(s_misc[2]), vI = static_cast<uint32_t>(s_misc[4]);
+      const uint32_t hi = kI > vI ? kI : vI;
+      for (uint32_t x = static_cast<uint32_t>(s_misc[3]); x < hi; ++x) {
+        if (x >= kI) mbar_arrive(bar(FULL + x % STAGES));
+        if (x >= vI) mbar_arrive(bar(FULL + x % STAGES));
         (void)mbar_wait_bounded(bar(FULL + x % STAGES), (x / STAGES) & 1u);
+      }
     }
     __syncthreads();
   }
   if (warp == kTcMmaWarp) {
     tc_fence_after_sync();
-    tmem_dealloc(tmem, kTmemCols);
+    tmem_dealloc(static_cast<uint32_t>(s_misc[0]), kTmemCols);
   }
-
 }
 
 // --------------------------------------------------------------------------
@@ -698,7 +730,8 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
 // --------------------------------------------------------------------------
 using TcKernelFn = void (*)(const CUtensorMap, const CUtensorMap, const AttnParams);
 
-// Lanes per query row: as many as 128 TMEM lanes allow, at most 4.
+// Copies of each query row (lanes per row): as many as 128 TMEM lanes allow,
+// at most 4.
 static int tc_key_split(int R) { return R <= 32 ? 4 : (R <= 64 ? 2 : 1); }
 
 template <int D>
@@ -709,9 +742,18 @@ static TcKernelFn tc_kernel(int F) {
   return verify_attention_tc_kernel<D, S, 1>;
 }
 
-int tc_smem_bytes(int head_dim, int B) {
-  if (head_dim == 128) return TcSmem<128, TcConfig<128>::kStages>::bytes(B);
-  if (head_dim == 64) return TcSmem<64, TcConfig<64>::kStages>::bytes(B);
+template <int D>
+static int tc_bytes(int F, int B) {
+  constexpr int S = TcConfig<D>::kStages;
+  if (F == 4) return TcSmem<D, S, 4>::bytes(B);
+  if (F == 2) return TcSmem<D, S, 2>::bytes(B);
+  return TcSmem<D, S, 1>::bytes(B);
+}
+
+int tc_smem_bytes(int head_dim, int R, int B) {
+  const int F = tc_key_split(R);
+  if (head_dim == 128) return tc_bytes<128>(F, B);
+  if (head_dim == 64) return tc_bytes<64>(F, B);
   return 0;
 }
 
@@ -722,10 +764,13 @@ int tc_setup(int head_dim, int device) {
   const int k = head_dim == 128 ? 1 : 0;
   std::lock_guard<std::mutex> lock(mu);
   if (done[device][k]) return SF_OK;
-  const int smem = tc_smem_bytes(head_dim, SF_MAX_BATCH);
   for (int F : {1, 2, 4}) {
     TcKernelFn fn = head_dim == 128 ? tc_kernel<128>(F) : tc_kernel<64>(F);
+    const int smem = head_dim == 128 ? tc_bytes<128>(F, SF_MAX_BATCH) : tc_bytes<64>(F, SF_MAX_BATCH);
     cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    if (e == cudaSuccess)
+      e = cudaFuncSetAttribute(fn, cudaFuncAttributePreferredSharedMemoryCarveout,
+                               cudaSharedmemCarveoutMaxShared);
     if (e != cudaSuccess)
       return fail(SF_ERR_CUDA, "cudaFuncSetAttribute (tcgen05 kernel): %s", cudaGetErrorString(e));
   }

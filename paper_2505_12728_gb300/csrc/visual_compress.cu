@@ -156,14 +156,22 @@ compress_apply_kernel(const __grid_constant__ CUtensorMap tmap_f, const __grid_c
     s_misc[2] = 0;
     s_misc[3] = 0;
   }
-  if (warp == kVcMmaWarp) {
-    tmem_alloc(smem_addr(s_misc), p.tmem_cols);
-    tmem_relinquish_alloc_permit();
-    tc_fence_before_sync();
+  __syncthreads();  // barrier initialisation visible to every role
+  // Tensor memory only once the previous kernel on the stream has completed
+  // (a predecessor still waiting for its own predecessor may not have
+  // allocated yet; holding TMEM here could deadlock the pair).
+  uint32_t tmem = 0;
+  if (warp != kVcProducerWarp) {
+    if (warp == kVcMmaWarp) {
+      grid_dependency_wait();
+      tmem_alloc(smem_addr(s_misc), p.tmem_cols);
+      tmem_relinquish_alloc_permit();
+      tc_fence_before_sync();
+    }
+    named_bar_sync(3, 160);
+    tc_fence_after_sync();
+    tmem = static_cast<uint32_t>(s_misc[0]);
   }
-  __syncthreads();
-  tc_fence_after_sync();
-  const uint32_t tmem = static_cast<uint32_t>(s_misc[0]);
 
   if (warp == kVcProducerWarp) {
     if (lane == 0) {
