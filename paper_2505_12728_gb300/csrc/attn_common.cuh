@@ -21,9 +21,7 @@ struct AttnParams {
   __nv_bfloat16 *out;
   float *lse;
   uint32_t *status;
-  int2 *seg_desc;     // [B * H_kv]: {first CTA, pieces} of each segment
   uint32_t *tickets;  // [2 * B * H_kv], zero between calls (in-kernel merges)
-  int merge_in_kernel;  // 1: last CTA of a segment merges; 0: merge kernel
   int cs;             // CTAs per cluster of the launch (1: no clusters)
   int push;           // cluster mode: peers push partial rows into the merging CTA
   int push_off;       // byte offset of the push area in dynamic shared memory
@@ -242,7 +240,7 @@ __device__ __forceinline__ void merge_one(const float *part0, size_t stride, int
 int tc_smem_bytes(int head_dim, int R, int B);
 // Raises the kernel's shared-memory limit once per device.
 int tc_setup(int head_dim, int device);
-// Launches the tcgen05 split kernel over G CTAs.
+// Launches the tcgen05 split kernel over G CTAs, then its merge kernel.
 int tc_launch(int head_dim, int G, int smem, const CUtensorMap &tk, const CUtensorMap &tv,
               const AttnParams &prm, cudaStream_t stream);
 

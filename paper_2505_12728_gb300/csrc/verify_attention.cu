@@ -35,8 +35,8 @@
 //        memory and merge them through distributed shared memory;
 //      - otherwise the CTA that takes the last ticket of the segment (an
 //        atomic counter; nobody waits) merges the fp32 partials;
-//      - the tcgen05 kernel's split segments (many rows): verify_merge_kernel,
-//        one thread per output quad.
+//      - the tcgen05 kernel's split segments (many rows, larger partials):
+//        verify_tc_merge_kernel, spread over the whole GPU.
 //  * Launches use programmatic stream serialisation: the partition, the
 //    block-table reads (for one sequence, its whole row copied to shared
 //    memory next to the seq_lens read) and the first copies of prefix tiles
@@ -285,7 +285,6 @@ verify_attention_kernel(const __grid_constant__ CUtensorMap tmap_k,
       waited = true;
     }
     issue_prologue(pre, prologue);
-    if (lt0 == 0 && tid == 0) p.seg_desc[seg] = make_int2(c_first, aligned ? 1 : n_pieces);
     seg_b = b;
     seg_h = h_kv;
 
@@ -661,8 +660,6 @@ verify_attention_kernel(const __grid_constant__ CUtensorMap tmap_k,
         }
       }
     }
-    if (!p.merge_in_kernel) continue;  // verify_merge_kernel combines the pieces
-
     // ---- few rows: the last CTA of the segment to finish merges it ----
     __threadfence();
     __syncthreads();
@@ -774,53 +771,6 @@ verify_attention_kernel(const __grid_constant__ CUtensorMap tmap_k,
   }
 }
 
-// Merge for shapes with many rows per KV head (GQA): the pieces of every
-// split segment are combined by a grid-stride loop with one item per 4
-// output columns of a row, in piece order (deterministic):
-//   M = max_q m_q,  L = sum_q l_q 2^(m_q - M),  O = sum_q 2^(m_q - M) O_q / L,
-//   lse = (M + log2 L) ln 2.
-// Pieces are read in batches of kMergeBatchGqa with a running (online)
-// rescale, so a batch costs one memory round trip.  Launched right after the
-// split kernel with programmatic stream serialisation: its CTAs are
-// scheduled while the split grid runs and wait for it before reading
-// anything.  At most 64 registers per thread, so that several of its CTAs
-// fit next to a split CTA and the whole grid is resident (and has let the
-// next kernel be scheduled) before the split grid completes.
-constexpr int kMergeThreads = 128;
-constexpr int kMergeBatchGqa = 8;
-
-template <int D>
-__global__ void __launch_bounds__(kMergeThreads, 8)
-verify_merge_kernel(const __grid_constant__ AttnParams p) {
-  constexpr float kLn2 = 0.6931471805599453f;
-  constexpr int C4 = D / 4;                       // items per row
-  grid_launch_dependents();
-  grid_dependency_wait();
-  const int per_seg = p.R * C4;
-  const long long total = (long long)per_seg * p.B * p.H_kv;
-  const size_t stride = (size_t)p.slot_stride;
-  for (long long item = (long long)blockIdx.x * kMergeThreads + threadIdx.x; item < total;
-       item += (long long)gridDim.x * kMergeThreads) {
-    const int seg = static_cast<int>(item / per_seg);
-    const int rem = static_cast<int>(item % per_seg);
-    const int r = rem / C4, c4 = rem % C4;
-    const int2 desc = p.seg_desc[seg];            // {first CTA, pieces}
-    if (desc.y <= 1) continue;                    // the split kernel wrote it
-    float4 ov;
-    float M, Ls;
-    merge_one<D, false, kMergeBatchGqa>(p.partials + (size_t)(desc.x + seg) * stride, stride, p.R,
-                                        r, c4, desc.y, ov, M, Ls);
-    const int b = seg / p.H_kv, h_kv = seg % p.H_kv;
-    const int i = r / p.group, j = r % p.group;
-    const size_t row = ((size_t)b * p.n_q + i) * p.H_q + (size_t)h_kv * p.group + j;
-    uint2 packed;
-    packed.x = pack_bf16x2(ov.x, ov.y);
-    packed.y = pack_bf16x2(ov.z, ov.w);
-    *reinterpret_cast<uint2 *>(p.out + row * D + 4 * c4) = packed;
-    if (p.lse && c4 == 0) p.lse[row] = (M + log2f(Ls)) * kLn2;
-  }
-}
-
 // --------------------------------------------------------------------------
 // host side
 // --------------------------------------------------------------------------
@@ -857,14 +807,13 @@ static AttnVariant select_variant(int D) {
 }
 
 struct AttnLayout {
-  size_t desc_off, tickets_off, partials_off, total;
+  size_t tickets_off, partials_off, total;
 };
 
 static AttnLayout attn_layout(int B, int H_kv, int R, int D, long long G) {
   AttnLayout l;
   const size_t segs = (size_t)B * H_kv;
-  l.desc_off = 256;
-  l.tickets_off = round_up(l.desc_off + 8 * segs, 256);
+  l.tickets_off = 256;
   l.partials_off = round_up(l.tickets_off + 8 * segs, 256);
   l.total = round_up(l.partials_off + (size_t)(G + (long long)segs) * partial_slot_floats(R, D) * 4,
                      256);
@@ -1148,7 +1097,7 @@ int sf_verify_attention_kernel_launches(int B, int n_q, int H_q, int H_kv, int h
   sf::AttnPlan plan;
   if (sf::plan_attention(B, n_q, H_q, H_kv, head_dim, max_pages_per_seq, num_splits, &plan) != SF_OK)
     return 0;
-  return plan.tc ? 2 : 1;  // the tcgen05 kernel leaves its merge to verify_merge_kernel
+  return plan.tc ? 2 : 1;  // the tcgen05 split kernel is followed by its merge kernel
 }
 
 int sf_verify_attention(const void *q, const void *k_cache, const void *v_cache,
@@ -1189,12 +1138,7 @@ int sf_verify_attention(const void *q, const void *k_cache, const void *v_cache,
   prm.out = static_cast<__nv_bfloat16 *>(out);
   prm.lse = lse;
   prm.status = reinterpret_cast<uint32_t *>(ws);
-  prm.seg_desc = reinterpret_cast<int2 *>(ws + lay.desc_off);
   prm.tickets = reinterpret_cast<uint32_t *>(ws + lay.tickets_off);
-  // One row tile (MHA, n_q <= 16): the partials are small and the last CTA
-  // of a segment merges them without a second launch.  More rows (GQA): a
-  // grid-wide merge kernel spreads the larger partials over many SMs.
-  prm.merge_in_kernel = R <= 16 ? 1 : 0;
   prm.cs = plan.cs;
   prm.push = plan.push;
   prm.push_off = plan.push_off;
@@ -1240,15 +1184,6 @@ int sf_verify_attention(const void *q, const void *k_cache, const void *v_cache,
     e = cudaLaunchKernelEx(&cfg, plan.v.fn, tk, tv, prm);
     if (e != cudaSuccess) return fail(SF_ERR_CUDA, "verify attention launch: %s", cudaGetErrorString(e));
   }
-  if (prm.merge_in_kernel) return SF_OK;
-  const long long items = (long long)R * (head_dim / 4) * B * H_kv;
-  cfg.gridDim = dim3(static_cast<unsigned>((items + kMergeThreads - 1) / kMergeThreads));
-  cfg.blockDim = dim3(kMergeThreads);
-  cfg.dynamicSmemBytes = 0;
-  cfg.numAttrs = 1;  // programmatic serialisation only, no clusters
-  e = head_dim == 64 ? cudaLaunchKernelEx(&cfg, verify_merge_kernel<64>, prm)
-                     : cudaLaunchKernelEx(&cfg, verify_merge_kernel<128>, prm);
-  if (e != cudaSuccess) return fail(SF_ERR_CUDA, "verify merge launch: %s", cudaGetErrorString(e));
   return SF_OK;
 }
 
@@ -1328,9 +1263,9 @@ extern "C" int sf_verify_attention_noalloc(const void *q, const void *k_cache,
   void *scratch = nullptr;
   st = static_scratch_address(&scratch);
   if (st != SF_OK) return st;
-  // The status word and the merge tickets must start at zero; descriptors
-  // and partials are written before they are read.  The scratch keeps
-  // whatever the previous call left.
+  // The status word and the merge tickets must start at zero; partials are
+  // written before they are read.  The scratch keeps whatever the previous
+  // call left.
   cudaError_t e = cudaMemsetAsync(scratch, 0, lay.partials_off, stream);
   if (e != cudaSuccess) return fail(SF_ERR_CUDA, "clearing the scratch: %s", cudaGetErrorString(e));
   return sf_verify_attention(q, k_cache, v_cache, block_table, seq_lens, B, n_q, H_q, H_kv,

@@ -5,8 +5,7 @@
 // It computes exactly what the mma.sync kernel in verify_attention.cu
 // computes (Sec. 3.1: the K draft tokens are scored in one forward pass, so
 // each of the n_q new rows attends to the prefix plus the causal draft
-// block), with the same fp32 partial format, so verify_merge_kernel combines
-// split segments.  Design points:
+// block).  Design points:
 //  * One CTA per SM with a six-stage ring (192 KB): the prefix tiles of the
 //    ring are copied before griddepcontrol.wait, so they land while the
 //    previous kernel on the stream finishes.  Tensor memory (all 512
@@ -54,8 +53,11 @@
 //    divided by (rows with a handful of visible keys would otherwise show
 //    P's bf16 rounding).
 //  * A piece that covers a whole segment writes bf16 out and the LSE; a
-//    split segment's pieces write fp32 partials to the workspace, which the
-//    merge kernel of verify_attention.cu combines.
+//    split segment's pieces write fp32 partials to the workspace (O as
+//    [D/4][R] float4, so that a warp's stores are contiguous), which
+//    verify_tc_merge_kernel combines across the whole GPU right after this
+//    kernel (one CTA merging a segment's ~250 KB of partials alone took
+//    longer than the whole split phase).
 //  * K/V copies run before griddepcontrol.wait only for tiles that lie
 //    wholly in the prefix; tiles holding draft positions
 //    (which the previous kernel on the stream may have just written) are
@@ -86,9 +88,11 @@ constexpr float kRescaleLog2 = 8.f;
 // this many tiles above the balanced share (a second piece in a CTA costs
 // about that much: another Q load, epilogue and pipeline start).
 constexpr int kAlignSlackTiles = 3;
-// Registers per thread: low enough that several merge-kernel CTAs fit next
-// to a split CTA on its SM.
-constexpr int kTcMaxRegs = 168;
+// Registers per thread: low enough that a merge-kernel CTA (launched early,
+// waiting for this grid) fits next to a split CTA -- registers are
+// partitioned per SM sub-partition (16K each), and warps w and w + 4 of
+// both CTAs share one.
+constexpr int kTcMaxRegs = 128;
 constexpr int kTcNamedTmem = 1;     // softmax warps + MMA warp: TMEM allocated
 constexpr int kTcNamedSoftmax = 2;  // softmax warps: epilogue exchange
 
@@ -130,6 +134,80 @@ __device__ __forceinline__ void tmem_st_cols(uint32_t taddr, const uint32_t (&v)
   if constexpr (N == 32) tmem_st_32x32b_x32(taddr, v);
   else if constexpr (N == 16) tmem_st_32x32b_x16(taddr, v);
   else tmem_st_32x32b_x8(taddr, v);
+}
+
+// The work partition of the split kernel, decided identically by every CTA
+// (of the split kernel and of its merge kernel) from seq_lens:
+//  * balanced: the batch's tiles in one ordered list cut into G equal
+//    ranges (a CTA may hold pieces of several segments);
+//  * segment-aligned: segment s gets ceil(tiles_s / Ta) CTAs and every CTA
+//    holds one piece, with the smallest Ta whose pieces fit the grid --
+//    chosen when Ta is close to the balanced share.
+// s_prefix holds the exclusive prefix of per-sequence tile counts
+// (tile_prefix); s_cpre receives, for the aligned partition, the first CTA
+// of each sequence; s_scratch is one int per warp.  Every thread calls it.
+struct TcPartition {
+  TilePartition part;  // the balanced partition (also defines Tot and G)
+  bool aligned;
+  int Ta;
+};
+
+template <int NT>
+__device__ TcPartition tc_partition(const AttnParams &p, const int *s_prefix, int *s_cpre,
+                                    int *s_scratch) {
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const uint32_t Tot = static_cast<uint32_t>(p.H_kv) * static_cast<uint32_t>(s_prefix[p.B]);
+  const int G = Tot < static_cast<uint32_t>(p.G) ? static_cast<int>(Tot) : p.G;
+  TcPartition tp;
+  tp.part = TilePartition{Tot, static_cast<uint32_t>(G), Tot / G, Tot % G};
+  tp.aligned = false;
+  tp.Ta = 0;
+  const int S = p.B * p.H_kv;
+  if (p.G > S) {
+    int Ta = static_cast<int>((Tot + static_cast<uint32_t>(p.G - S) - 1) / static_cast<uint32_t>(p.G - S));
+    const int Tmin = static_cast<int>((Tot + p.G - 1) / p.G);
+    tp.aligned = Ta <= Tmin + kAlignSlackTiles;
+    // the smallest piece length whose pieces still fit the grid (Ta always
+    // does: each segment's ceiling adds less than one CTA)
+    for (int cand = Tmin; tp.aligned && cand < Ta; ++cand) {
+      int local = 0;
+      for (int b = tid; b < p.B; b += NT) local += (s_prefix[b + 1] - s_prefix[b] + cand - 1) / cand;
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) local += __shfl_xor_sync(0xffffffffu, local, o);
+      if (lane == 0) s_scratch[warp] = local;
+      __syncthreads();
+      int need = 0;
+      for (int w = 0; w < NT / 32; ++w) need += s_scratch[w];
+      __syncthreads();
+      if (static_cast<long long>(need) * p.H_kv <= p.G) {
+        Ta = cand;
+        break;
+      }
+    }
+    tp.Ta = Ta;
+  }
+  if (tp.aligned) {
+    aligned_prefix<NT>(p, s_prefix, tp.Ta, s_cpre, s_scratch);
+    __syncthreads();
+  }
+  return tp;
+}
+
+// First CTA and number of pieces of segment (b, h) under partition tp.
+__device__ __forceinline__ void tc_segment(const TcPartition &tp, const AttnParams &p,
+                                           const int *s_prefix, const int *s_cpre, int b, int h,
+                                           int &c_first, int &n_pieces) {
+  const int tiles_b = s_prefix[b + 1] - s_prefix[b];
+  if (tp.aligned) {
+    const int ns = (tiles_b + tp.Ta - 1) / tp.Ta;
+    c_first = s_cpre[b] + h * ns;
+    n_pieces = ns;
+  } else {
+    const uint32_t first = static_cast<uint32_t>(p.H_kv) * static_cast<uint32_t>(s_prefix[b]) +
+                           static_cast<uint32_t>(h * tiles_b);
+    c_first = static_cast<int>(tp.part.owner(first));
+    n_pieces = static_cast<int>(tp.part.owner(first + tiles_b - 1)) - c_first + 1;
+  }
 }
 
 template <int D, int STAGES, int F>
@@ -193,28 +271,15 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
   tile_prefix<kTcThreads>(p, s_prefix, s_len, s_misc + 8);
   __syncthreads();
 
-  // Work partition, decided identically by every CTA from seq_lens:
-  //  * balanced: the batch's tiles in one ordered list cut into G equal
-  //    ranges (a CTA may hold pieces of several segments);
-  //  * segment-aligned: segment s gets ceil(tiles_s / Ta) CTAs, Ta =
-  //    ceil(Tot / (G - S)) so that they number at most G, and every CTA holds
-  //    one piece -- chosen when Ta is close to the balanced share.
-  // CTAs beyond the work get an empty range.
-  const uint32_t Tot = static_cast<uint32_t>(p.H_kv) * static_cast<uint32_t>(s_prefix[p.B]);
-  const int G = Tot < static_cast<uint32_t>(p.G) ? static_cast<int>(Tot) : p.G;
-  const TilePartition part{Tot, static_cast<uint32_t>(G), Tot / G, Tot % G};
-  const int S = p.B * p.H_kv;
-  bool aligned = false;
-  int Ta = 0;
-  if (p.G > S) {
-    Ta = static_cast<int>((Tot + static_cast<uint32_t>(p.G - S) - 1) / static_cast<uint32_t>(p.G - S));
-    aligned = Ta <= static_cast<int>((Tot + p.G - 1) / p.G) + kAlignSlackTiles;
-  }
+  const TcPartition tp = tc_partition<kTcThreads>(p, s_prefix, s_cpre, s_misc + 8);
+  const TilePartition &part = tp.part;
+  const bool aligned = tp.aligned;
+  const int Ta = tp.Ta;
+  const uint32_t Tot = part.Tot;
+  const int G = static_cast<int>(part.G);
   Piece apc{};  // the aligned partition's piece of this CTA
   uint32_t t_begin = Tot, t_end = Tot;
   if (aligned) {
-    aligned_prefix<kTcThreads>(p, s_prefix, Ta, s_cpre, s_misc + 8);
-    __syncthreads();
     const int c = static_cast<int>(blockIdx.x);
     if (c < s_cpre[p.B]) {
       int lo = 0, hi = p.B - 1;  // last sequence whose first CTA is <= c
@@ -456,15 +521,17 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
     auto q_row = [&](const Piece &pc) -> const __nv_bfloat16 * {
       return p.q + (((size_t)pc.b * p.n_q + qi) * p.H_q + (size_t)pc.h_kv * p.group + qj) * D;
     };
-    // this lane's Q row of piece pc into TMEM (zeros for padding rows)
-    auto load_q = [&](const Piece &pc, uint32_t tl) {
-      uint32_t qw[kQWords];
+    // this lane's Q row of piece pc (zeros for padding rows) into registers,
+    // then into TMEM
+    auto fetch_q = [&](const Piece &pc, uint32_t (&qw)[kQWords]) {
       const uint4 *src = reinterpret_cast<const uint4 *>(q_row(pc));
 #pragma unroll
       for (int u = 0; u < D / 8; ++u) {
         const uint4 v = valid ? __ldg(src + u) : make_uint4(0u, 0u, 0u, 0u);
         qw[4 * u] = v.x; qw[4 * u + 1] = v.y; qw[4 * u + 2] = v.z; qw[4 * u + 3] = v.w;
       }
+    };
+    auto store_q = [&](const uint32_t (&qw)[kQWords], uint32_t tl) {
 #pragma unroll
       for (int c = 0; c < kQWords; c += 32) {
         uint32_t part[32];
@@ -483,11 +550,17 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
       }
     }
     grid_dependency_wait();
-    named_bar_sync(kTcNamedTmem, kTcSoftmaxThreads + 32);
-    tc_fence_after_sync();
+    {
+      // the Q loads are in flight while the MMA warp allocates TMEM
+      uint32_t qw[kQWords];
+      if (t_begin < t_end) fetch_q(pc0, qw);
+      named_bar_sync(kTcNamedTmem, kTcSoftmaxThreads + 32);
+      tc_fence_after_sync();
+      const uint32_t tl0 = static_cast<uint32_t>(s_misc[0]) + (static_cast<uint32_t>(warp * 32) << 16);
+      if (t_begin < t_end) store_q(qw, tl0);
+    }
     const uint32_t tmem = static_cast<uint32_t>(s_misc[0]);
     const uint32_t tl = tmem + (static_cast<uint32_t>(warp * 32) << 16);
-    if (t_begin < t_end) load_q(pc0, tl);
     tmem_wait_st();
     tc_fence_before_sync();
     mbar_arrive(bar(QFULL));
@@ -498,7 +571,6 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
     for (uint32_t t = t_begin; t < t_end; ++pi) {
       const Piece pc = pi == 0 ? pc0 : piece_at(t);
       t += pc.n_tiles;
-      if (pc.lt0 == 0 && tid == 0) p.seg_desc[pc.seg] = make_int2(pc.c_first, pc.n_pieces);
       if (t < t_end) {
         // the next piece's Q rows into L2 (read after this piece's tiles)
         const Piece nx = piece_at(t);
@@ -608,7 +680,9 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
       // its last score tile was read above), so that the next piece's first
       // Q K^T overlaps this epilogue ----
       if (ok && t < t_end) {
-        load_q(piece_at(t), tl);
+        uint32_t qw[kQWords];
+        fetch_q(piece_at(t), qw);
+        store_q(qw, tl);
         tmem_wait_st();
         tc_fence_before_sync();
         mbar_arrive(bar(QFULL));
@@ -680,10 +754,11 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
             dst[q4] = wv;
           }
         } else if (writer) {
-          float4 *dst = reinterpret_cast<float4 *>(part0 + (size_t)r * D + ch * 32);
+          // [D/4][R] float4: the warp's 32 rows of one quad are contiguous
+          float4 *dst = reinterpret_cast<float4 *>(part0) + (size_t)(ch * 8) * p.R + r;
 #pragma unroll
           for (int q4 = 0; q4 < 8; ++q4)
-            dst[q4] = make_float4(o[4 * q4], o[4 * q4 + 1], o[4 * q4 + 2], o[4 * q4 + 3]);
+            dst[(size_t)q4 * p.R] = make_float4(o[4 * q4], o[4 * q4 + 1], o[4 * q4 + 2], o[4 * q4 + 3]);
         }
         if constexpr (F > 1) named_bar_sync(kTcNamedSoftmax, kTcSoftmaxThreads);
       }
@@ -722,6 +797,93 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
   if (warp == kTcMmaWarp) {
     tc_fence_after_sync();
     tmem_dealloc(static_cast<uint32_t>(s_misc[0]), kTmemCols);
+  }
+}
+
+// --------------------------------------------------------------------------
+// Merge of split segments, one CTA per SM (256 threads).  Before the
+// dependency wait every CTA recomputes the split kernel's partition from
+// seq_lens, so that after it only the partials are read: one item per output
+// quad (row r, columns 4c4 .. 4c4+3) of every split segment, consecutive
+// threads on consecutive rows of one quad (the [D/4][R] slots make a warp's
+// loads contiguous), with the loads of kTcMergeBatch pieces in flight at
+// once.  In piece order (deterministic):
+//   M = max_q m_q,  L = sum_q l_q 2^(m_q - M),  O = sum_q 2^(m_q - M) O_q / L,
+//   lse = (M + log2 L) ln 2.
+// Launched right after the split kernel with programmatic stream
+// serialisation: its CTAs are resident while the split grid runs.
+// --------------------------------------------------------------------------
+constexpr int kTcMergeThreads = 256;
+constexpr int kTcMergeBatch = 12;
+// 256 threads x 104 registers fit next to a split CTA (224 x 128) on one SM
+constexpr int kTcMergeMaxRegs = 104;
+
+template <int D>
+__global__ void __maxnreg__(kTcMergeMaxRegs)
+verify_tc_merge_kernel(const __grid_constant__ AttnParams p) {
+  constexpr float kLn2 = 0.6931471805599453f;
+  constexpr int C4 = D / 4;
+  extern __shared__ int s_arr[];
+  __shared__ int s_scratch[16];
+  int *s_prefix = s_arr;             // [B+1]
+  int *s_len = s_prefix + p.B + 1;   // [B]
+  int *s_cpre = s_len + p.B;         // [B+1]
+  grid_launch_dependents();
+  tile_prefix<kTcMergeThreads>(p, s_prefix, s_len, s_scratch + 8);
+  __syncthreads();
+  const TcPartition tp = tc_partition<kTcMergeThreads>(p, s_prefix, s_cpre, s_scratch + 8);
+  grid_dependency_wait();
+  const int per_seg = p.R * C4;
+  const long long total = (long long)per_seg * p.B * p.H_kv;
+  const size_t stride = (size_t)p.slot_stride;
+  for (long long item = (long long)blockIdx.x * kTcMergeThreads + threadIdx.x; item < total;
+       item += (long long)gridDim.x * kTcMergeThreads) {
+    const int seg = static_cast<int>(item / per_seg);
+    const int rem = static_cast<int>(item % per_seg);
+    const int c4 = rem / p.R, r = rem % p.R;
+    const int b = seg / p.H_kv, h_kv = seg % p.H_kv;
+    int c_first, n_pieces;
+    tc_segment(tp, p, s_prefix, s_cpre, b, h_kv, c_first, n_pieces);
+    if (n_pieces <= 1) continue;  // the split kernel wrote the output
+    const float *slot0 = p.partials + (size_t)(c_first + seg) * stride;
+    float M = -INFINITY, Ls = 0.f;
+    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+    for (int q0 = 0; q0 < n_pieces; q0 += kTcMergeBatch) {
+      float mv[kTcMergeBatch], lv[kTcMergeBatch];
+      float4 xv[kTcMergeBatch];
+#pragma unroll
+      for (int u = 0; u < kTcMergeBatch; ++u) {
+        const bool in = q0 + u < n_pieces;
+        const float *slot = slot0 + (size_t)(q0 + u) * stride;
+        mv[u] = in ? slot[(size_t)p.R * D + r] : -INFINITY;
+        lv[u] = in ? slot[(size_t)p.R * D + p.R + r] : 0.f;
+        xv[u] = in ? reinterpret_cast<const float4 *>(slot)[(size_t)c4 * p.R + r]
+                   : make_float4(0.f, 0.f, 0.f, 0.f);
+      }
+      float Mb = M;
+#pragma unroll
+      for (int u = 0; u < kTcMergeBatch; ++u) Mb = fmaxf(Mb, mv[u]);
+      // weights 2^(m - Mb) <= 1 (fast_exp2(-inf) = 0: pieces without a
+      // visible key for this row, and the empty running state of the first batch)
+      const float a = fast_exp2(M - Mb);
+      Ls *= a;
+      acc.x *= a; acc.y *= a; acc.z *= a; acc.w *= a;
+#pragma unroll
+      for (int u = 0; u < kTcMergeBatch; ++u) {
+        const float w = fast_exp2(mv[u] - Mb);
+        Ls += lv[u] * w;
+        acc.x += xv[u].x * w; acc.y += xv[u].y * w; acc.z += xv[u].z * w; acc.w += xv[u].w * w;
+      }
+      M = Mb;
+    }
+    const int i = r / p.group, j = r % p.group;
+    const size_t row = ((size_t)b * p.n_q + i) * p.H_q + (size_t)h_kv * p.group + j;
+    const float inv = 1.f / Ls;
+    uint2 packed;
+    packed.x = pack_bf16x2(acc.x * inv, acc.y * inv);
+    packed.y = pack_bf16x2(acc.z * inv, acc.w * inv);
+    *reinterpret_cast<uint2 *>(p.out + row * D + 4 * c4) = packed;
+    if (p.lse && c4 == 0) p.lse[row] = (M + log2f(Ls)) * kLn2;
   }
 }
 
@@ -794,6 +956,15 @@ int tc_launch(int head_dim, int G, int smem, const CUtensorMap &tk, const CUtens
   TcKernelFn fn = head_dim == 128 ? tc_kernel<128>(F) : tc_kernel<64>(F);
   cudaError_t e = cudaLaunchKernelEx(&cfg, fn, tk, tv, prm);
   if (e != cudaSuccess) return fail(SF_ERR_CUDA, "verify attention (tcgen05) launch: %s", cudaGetErrorString(e));
+  const long long items = (long long)prm.R * (head_dim / 4) * prm.B * prm.H_kv;
+  long long ctas = (items + kTcMergeThreads - 1) / kTcMergeThreads;
+  if (ctas > G) ctas = G;  // one per SM (G is the SM count unless num_splits asks for fewer)
+  cfg.gridDim = dim3(static_cast<unsigned>(ctas));
+  cfg.blockDim = dim3(kTcMergeThreads);
+  cfg.dynamicSmemBytes = 4 * (3 * prm.B + 2);
+  e = head_dim == 64 ? cudaLaunchKernelEx(&cfg, verify_tc_merge_kernel<64>, prm)
+                     : cudaLaunchKernelEx(&cfg, verify_tc_merge_kernel<128>, prm);
+  if (e != cudaSuccess) return fail(SF_ERR_CUDA, "verify merge launch: %s", cudaGetErrorString(e));
   return SF_OK;
 }
 

@@ -239,7 +239,7 @@ def test_one_sequence_block_table_row_widths(oracle_mod, prefix, max_pages):
 
 def test_kernel_launch_counts_follow_the_rows_per_kv_head():
     # at most 16 rows per KV head: one launch (the split kernel merges in
-    # place); more: the tcgen05 split kernel and the merge kernel
+    # place); more: the tcgen05 split kernel and its merge kernel
     assert sfv.verify_attention_kernel_launches(1, 5, 32, 32, 128, 189) == 1
     assert sfv.verify_attention_kernel_launches(2, 16, 8, 8, 64, 40) == 1
     assert sfv.verify_attention_kernel_launches(4, 8, 28, 4, 128, 305) == 2
