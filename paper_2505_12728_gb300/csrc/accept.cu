@@ -11,26 +11,27 @@
 // x_i is the argmax of row i, and emit the argmax of row j.
 //
 // GB300 design.  The whole cost is streaming the (k+1) x V fp32 logits once
-// (plus one row of q for the draw), so both kernels are coalesced 128-bit
-// streaming reductions spread over many CTAs, with no tensor cores, and the
-// critical path is a short chain of memory round trips:
-//  * accept_stats_kernel, grid (chunks, k+1, B): each CTA reduces a chunk of
-//    one row to (max, first argmax, sum exp((x - max)/tau)) with the chunk in
-//    registers; the CTA whose chunk holds the row's draft token also records
-//    that token's logit and draft probability.  The last CTA of a sequence
-//    to finish (one atomic ticket; nobody waits) combines every row, one warp
-//    per row, and takes the k accept/reject decisions (float-float, below).
-//  * accept_draw_kernel, grid (chunks, B), launched with programmatic stream
-//    serialisation so that it is resident while the first kernel drains: for
-//    sampled sequences each CTA sums the residual (or bonus) mass of a chunk
-//    of row j; the last CTA of the sequence locates the chunk holding u_k * S
-//    with a float-float scan over chunk sums and scans that chunk in
-//    ascending token order.
-// Arithmetic: per-element terms are fp32 (expf, explicitly rounded products
-// and differences, identical wherever a value is recomputed); sums, scans and
-// the accept tests use float-float numbers (an unevaluated sum hi + lo of two
-// fp32 values, ~44 significant bits) built from exactly rounded fp32
-// operations, accumulated in a fixed order (results are deterministic).
+// (plus one row of q for the draw), so every kernel is a coalesced 128-bit
+// streaming reduction spread over many CTAs, with no tensor cores, and the
+// critical path is a short chain of memory round trips.  Three launch plans:
+//  * V <= 16 x 2048: accept_cluster_kernel, one thread-block cluster per
+//    sequence, the phases separated by cluster barriers (below);
+//  * larger V: accept_chunks_kernel (every row in 1024-token chunks over
+//    all SMs, row records combined by the warp that completes a row) then
+//    accept_finish_kernel (decisions, then the residual draw in C2 chunks of
+//    row j, the last CTA of a sequence scanning for u_k * S);
+//  * behind the fused LM head, whose projection already left per-CTA row
+//    statistics: accept_decide_kernel then accept_draw_kernel.
+// Every launch uses programmatic stream serialisation: a kernel is resident
+// while the previous one drains and waits for it (griddepcontrol.wait)
+// before reading its results.
+// Arithmetic: per-element terms are fp32 (2^x by the hardware approximation
+// of explicitly rounded differences and products; the decisions' p(x) by
+// expf on a float-float difference; a term recomputed within a draw is
+// recomputed identically); sums, scans and the accept tests use float-float
+// numbers (an unevaluated sum hi + lo of two fp32 values, ~44 significant
+// bits) built from exactly rounded fp32 operations, accumulated in a fixed
+// order (results are deterministic).
 // GB300's fp64 pipe is far too slow for this latency-bound path, and
 // float-float gives the accuracy the decisions need.
 #include <climits>
@@ -45,24 +46,15 @@ namespace sf {
 
 constexpr int kAccThreads = kFfThreads;
 constexpr int kAccWarps = kFfWarps;
-constexpr int kMaxPerThread = 32;                       // elements held per thread
-constexpr int kMaxChunk = kAccThreads * kMaxPerThread;  // 8192 elements per CTA
+// Rows are cut into segments of 1024 tokens (a warp, eight float4 per lane):
+// the unit of the chunk records and of the draw's partial sums.
+constexpr int kSegTokens = 1024;
 
 
-struct ChunkRec {  // one chunk of one target row
-  float m;         // largest raw logit in the chunk
+struct alignas(16) RowStat {  // a target row, or a run of its chunks (one 16-byte load)
+  float m;         // largest raw logit
   int arg;         // its first index
-  ff S;            // sum of exp((x - m) / tau) over the chunk; 0 for greedy rows
-  float lx;        // logit of the row's draft token, if it lies in this chunk
-  float qx;        // its draft probability
-  int has_x;       // 1 if the row's draft token lies in this chunk
-  int pad;
-};
-
-struct RowStat {   // one combined target row
-  float m;
-  int arg;
-  ff S;
+  ff S;            // sum of exp((x - m) / tau); 0 for greedy rows
 };
 
 struct SeqState {
@@ -70,9 +62,9 @@ struct SeqState {
   int pad[3];
 };
 
-struct DrawPart {
-  ff sum_r;        // residual (or bonus) mass of the chunk
-  ff sum_p;        // target mass of the chunk (fallback when the residual is 0)
+struct alignas(16) DrawPart {  // one segment of row j
+  ff sum_r;        // residual (or bonus) mass of the segment
+  ff sum_p;        // target mass of the segment (fallback when the residual is 0)
   int last_r;      // last index with r > 0 (-1 if none)
   int last_p;      // last index with p > 0 (-1 if none)
   int pad[2];
@@ -88,15 +80,15 @@ struct AccParams {
   int32_t *out_tokens;     // [B][k+1]
   float *ratio;            // [B][k] or null
   uint32_t *status;
-  uint32_t *seq_tickets;   // [B]
   uint32_t *draw_tickets;  // [B]
-  ChunkRec *chunks;        // [B][k+1][C1]
+  RowStat *runs;           // [B][k+1][C1]: per row, one record per run of the chunk kernel
   RowStat *rows;           // [B][k+1]
   SeqState *seqs;          // [B]
-  DrawPart *parts;         // [B][C2]
+  DrawPart *parts;         // [B][C1]
   int B, k, V;
-  int C1, CV1;             // stats chunks per row, elements per chunk
-  int C2, CV2;             // draw chunks per row, elements per chunk
+  int C1;                  // segments per row: ceil(V / kSegTokens)
+  int C2;                  // draw CTAs per row: ceil(C1 / kAccWarps)
+  int NW1;                 // warps of the chunk kernel
   int vec4;                // rows are 16-byte aligned and V % 4 == 0
 };
 
@@ -129,14 +121,14 @@ __device__ __forceinline__ void draw_terms(float x, float qx, bool residual, flo
 __device__ void decide_sequence(const AccParams &p, int b, bool greedy, float tau, int my_tok,
                                 float my_u, const float *s_rm, const int *s_rarg, const ff *s_rS,
                                 const float *s_rlx, const float *s_rqx, const int *s_rhx,
-                                int *s_acc) {
+                                int *s_acc, bool write = true, int *s_j = nullptr) {
   const int tid = threadIdx.x, k = p.k, V = p.V;
   if (tid < k) {
     const int i = tid, x = my_tok;
     int acc = 0;
     float ratio = 0.f;
     if (x < 0 || x >= V || !s_rhx[i]) {
-      set_status(p.status, SF_DEVICE_BAD_TOKEN);  // treated as a rejection
+      if (write) set_status(p.status, SF_DEVICE_BAD_TOKEN);  // treated as a rejection
     } else if (greedy) {
       acc = (x == s_rarg[i]);
       ratio = acc ? 1.f : 0.f;
@@ -151,7 +143,7 @@ __device__ void decide_sequence(const AccParams &p, int b, bool greedy, float ta
       ratio = qd > 0.f ? fminf(1.f, __fdiv_rn(px, qd)) : 1.f;
     }
     s_acc[i] = acc;
-    if (p.ratio) p.ratio[(size_t)b * k + i] = ratio;
+    if (write && p.ratio) p.ratio[(size_t)b * k + i] = ratio;
   }
   __syncthreads();
   if (tid <= k) {
@@ -162,159 +154,15 @@ __device__ void decide_sequence(const AccParams &p, int b, bool greedy, float ta
     int32_t v = -1;
     if (tid < j) v = my_tok;
     else if (tid == j && greedy) v = s_rarg[j];
-    if (!(tid == j && !greedy)) p.out_tokens[(size_t)b * (k + 1) + tid] = v;
+    if (write && !(tid == j && !greedy)) p.out_tokens[(size_t)b * (k + 1) + tid] = v;
     if (tid == 0) {
-      p.num_accepted[b] = j;
-      p.seqs[b].j = j;
-    }
-  }
-}
-
-__global__ void __launch_bounds__(kAccThreads)
-accept_stats_kernel(const __grid_constant__ AccParams p) {
-  __shared__ ff s_d[32];
-  __shared__ float s_v[32];
-  __shared__ int s_i[32];
-  __shared__ int s_flag;
-  __shared__ int s_acc[SF_MAX_DRAFT];
-  __shared__ float s_rm[SF_MAX_DRAFT + 1], s_rlx[SF_MAX_DRAFT + 1], s_rqx[SF_MAX_DRAFT + 1];
-  __shared__ int s_rarg[SF_MAX_DRAFT + 1], s_rhx[SF_MAX_DRAFT + 1];
-  __shared__ ff s_rS[SF_MAX_DRAFT + 1];
-
-  // Every input (logits, q, tokens, uniforms, temperatures) may come from
-  // the previous kernel on the stream, which may let this grid start early:
-  // wait for it before reading anything.  Only then let the draw kernel be
-  // scheduled, so that it too starts after the previous kernel completed.
-  grid_dependency_wait();
-  grid_launch_dependents();
-
-  const int c = blockIdx.x, r = blockIdx.y, b = blockIdx.z;
-  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  const int k = p.k, V = p.V;
-  const float tau = p.tau[b];
-  const bool greedy = !(tau > 0.0f);
-  const float *row = p.logits + ((size_t)b * (k + 1) + r) * V;
-  const int c0 = c * p.CV1;
-  const int c1 = min(V, c0 + p.CV1);
-
-  // the row's draft token, and the decision inputs (used by the last CTA)
-  const int x_row = r < k ? p.tokens[(size_t)b * k + r] : -1;
-  int my_tok = -1;
-  float my_u = 0.f;
-  if (tid < k) {
-    my_tok = p.tokens[(size_t)b * k + tid];
-    my_u = p.u[(size_t)b * (k + 1) + tid];
-  }
-
-  // ---- chunk reduction: max / first argmax, then sum of exp ----
-  float vals[kMaxPerThread];
-  int n = 0;
-  float bv = -INFINITY;
-  int bi = INT_MAX;
-  if (p.vec4) {
-    const float4 *row4 = reinterpret_cast<const float4 *>(row);
-#pragma unroll
-    for (int t = 0; t < kMaxPerThread / 4; ++t) {
-      const int e = c0 + 4 * (tid + t * kAccThreads);
-      if (e < c1) {
-        const float4 x = row4[e / 4];
-        vals[4 * t + 0] = x.x; vals[4 * t + 1] = x.y; vals[4 * t + 2] = x.z; vals[4 * t + 3] = x.w;
-        if (better(x.x, e, bv, bi)) { bv = x.x; bi = e; }
-        if (better(x.y, e + 1, bv, bi)) { bv = x.y; bi = e + 1; }
-        if (better(x.z, e + 2, bv, bi)) { bv = x.z; bi = e + 2; }
-        if (better(x.w, e + 3, bv, bi)) { bv = x.w; bi = e + 3; }
-        n = 4 * t + 4;
+      if (write) {
+        p.num_accepted[b] = j;
+        p.seqs[b].j = j;
       }
-    }
-  } else {
-#pragma unroll
-    for (int t = 0; t < kMaxPerThread; ++t) {
-      const int e = c0 + tid + t * kAccThreads;
-      if (e < c1) {
-        const float x = row[e];
-        vals[t] = x;
-        if (better(x, e, bv, bi)) { bv = x; bi = e; }
-        n = t + 1;
-      }
+      if (s_j) *s_j = j;
     }
   }
-  // the CTA whose chunk holds the draft token records its logit and q
-  const bool has_x = x_row >= c0 && x_row < c1;
-  float lx = 0.f, qx = 0.f;
-  if (has_x && tid == 0) {
-    lx = row[x_row];
-    qx = p.q[((size_t)b * k + r) * V + x_row];
-  }
-  block_argmax(bv, bi, s_v, s_i);
-  ff S = ff_of(0.f);
-  if (!greedy && bv != -INFINITY) {
-    ff acc = ff_of(0.f);
-#pragma unroll
-    for (int t = 0; t < kMaxPerThread; t += 4) {
-      if (t < n) {
-        float e[4];
-#pragma unroll
-        for (int u = 0; u < 4; ++u) e[u] = t + u < n ? exp_scaled(vals[t + u], bv, tau) : 0.f;
-        acc = ff_add(acc, ff_of(sum4(e[0], e[1], e[2], e[3])));
-      }
-    }
-    S = block_sum(acc, s_d);
-  }
-
-  const size_t rowid = (size_t)b * (k + 1) + r;
-  if (tid == 0) p.chunks[rowid * p.C1 + c] = ChunkRec{bv, bi, S, lx, qx, has_x ? 1 : 0, 0};
-
-  // ---- the last CTA of the sequence combines every row and decides ----
-  __threadfence();
-  __syncthreads();
-  if (tid == 0)
-    s_flag = (atomicAdd(p.seq_tickets + b, 1u) == (unsigned)((k + 1) * p.C1 - 1)) ? 1 : 0;
-  __syncthreads();
-  if (!s_flag) return;
-  __threadfence();
-  for (int rr = warp; rr <= k; rr += kAccWarps) {
-    const ChunkRec *cr = p.chunks + ((size_t)b * (k + 1) + rr) * p.C1;
-    float mv = -INFINITY, rlx = 0.f, rqx = 0.f;
-    int mi = INT_MAX, hx = 0;
-    for (int cc = lane; cc < p.C1; cc += 32) {
-      const float cm = __ldcg(&cr[cc].m);
-      const int ca = __ldcg(&cr[cc].arg);
-      if (better(cm, ca, mv, mi)) { mv = cm; mi = ca; }
-      if (__ldcg(&cr[cc].has_x)) {
-        hx = 1;
-        rlx = __ldcg(&cr[cc].lx);
-        rqx = __ldcg(&cr[cc].qx);
-      }
-    }
-    warp_argmax(mv, mi);
-    const unsigned hmask = __ballot_sync(0xffffffffu, hx);
-    if (hmask) {
-      const int src = __ffs(hmask) - 1;
-      rlx = __shfl_sync(0xffffffffu, rlx, src);
-      rqx = __shfl_sync(0xffffffffu, rqx, src);
-    }
-    ff Sr = ff_of(0.f);
-    if (!greedy && mv != -INFINITY) {
-      for (int cc = lane; cc < p.C1; cc += 32) {
-        const ff cS = ff{__ldcg(&cr[cc].S.hi), __ldcg(&cr[cc].S.lo)};
-        if (ff_pos(cS))
-          Sr = ff_add(Sr, ff_mul(cS, exp_diff_accurate(__ldcg(&cr[cc].m), mv, tau)));
-      }
-      Sr = warp_sum_ff(Sr);
-    }
-    if (lane == 0) {
-      s_rm[rr] = mv;
-      s_rarg[rr] = mi;
-      s_rS[rr] = Sr;
-      s_rlx[rr] = rlx;
-      s_rqx[rr] = rqx;
-      s_rhx[rr] = hmask ? 1 : 0;
-      p.rows[(size_t)b * (k + 1) + rr] = RowStat{mv, mi, Sr};
-    }
-  }
-  __syncthreads();
-  decide_sequence(p, b, greedy, tau, my_tok, my_u, s_rm, s_rarg, s_rS, s_rlx, s_rqx, s_rhx, s_acc);
-  if (tid == 0) p.seq_tickets[b] = 0u;
 }
 
 // Single-kernel acceptance for V <= 16 * kClusterMaxSlice: one thread-block
@@ -691,173 +539,174 @@ accept_decide_kernel(const __grid_constant__ AccParams p, const SampStat *__rest
   decide_sequence(p, b, greedy, tau, my_tok, my_u, s_rm, s_rarg, s_rS, s_rlx, s_rqx, s_rhx, s_acc);
 }
 
-__global__ void __launch_bounds__(kAccThreads)
-accept_draw_kernel(const __grid_constant__ AccParams p) {
+// The residual (j < k) or bonus (j == k) draw of sequence b (grid (C2, B)
+// of kAccThreads threads; rs holds row j's max, argmax and sum).  Warp w of
+// CTA c sums the residual and target masses of segment c * kAccWarps + w of
+// row j (float-float) into its part; the last CTA of the sequence to finish
+// (one atomic ticket; nobody waits) locates the segment holding u_k * S with
+// a float-float scan over the segment sums in order, and scans that segment
+// in ascending token order, four tokens per thread.
+__device__ void draw_residual(const AccParams &p, int b, int c, int j, RowStat rs, float tau,
+                              float u_k) {
   __shared__ ff s_d[32];
-  __shared__ ff s_scan[32];
-  __shared__ float s_r[kMaxChunk];
-  __shared__ int s_flag, s_token, s_chunk, s_last;
+  __shared__ ff s_scan[kAccWarps + 1];
+  __shared__ int s_flag, s_seg, s_token;
   __shared__ ff s_base;
-
-  // The previous kernel (the statistics or decision kernel of this call)
-  // lets this grid start only after it has itself waited for the kernel
-  // before the call, so the call's inputs (temperature, uniforms) are in
-  // place already; j and the row statistics are waited for.
-  grid_launch_dependents();
-  const int c = blockIdx.x, b = blockIdx.y;
-  const int tid = threadIdx.x;
-  const int k = p.k, V = p.V;
-  const float tau = p.tau[b];
-  if (!(tau > 0.0f)) return;  // greedy sequences are complete
-  const float u_k = p.u[(size_t)b * (k + 1) + k];
-  grid_dependency_wait();     // j and the row statistics come from the previous kernel
-
-  const int j = __ldcg(&p.seqs[b].j);
-  const RowStat rs = {__ldcg(&p.rows[(size_t)b * (k + 1) + j].m),
-                      __ldcg(&p.rows[(size_t)b * (k + 1) + j].arg),
-                      ff{__ldcg(&p.rows[(size_t)b * (k + 1) + j].S.hi),
-                         __ldcg(&p.rows[(size_t)b * (k + 1) + j].S.lo)}};
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int k = p.k, V = p.V, NS = p.C1;
   const bool residual = j < k;
   const float invS = ff_div_to_f(1.0f, rs.S);
   const float *row = p.logits + ((size_t)b * (k + 1) + j) * V;
   const float *qrow = residual ? p.q + ((size_t)b * k + j) * V : nullptr;
-  const int c0 = c * p.CV2;
-  const int c1 = min(V, c0 + p.CV2);
+  DrawPart *parts = p.parts + (size_t)b * NS;
+  // four consecutive tokens from e (past V: logit -inf and q 0, terms 0)
+  auto load4 = [&](int e, float4 &x, float4 &qq) {
+    if (p.vec4) {
+      x = e < V ? *reinterpret_cast<const float4 *>(row + e)
+                : make_float4(-INFINITY, -INFINITY, -INFINITY, -INFINITY);
+      qq = (e < V && residual) ? __ldcs(reinterpret_cast<const float4 *>(qrow + e))
+                               : make_float4(0.f, 0.f, 0.f, 0.f);
+    } else {
+      x.x = e < V ? row[e] : -INFINITY;
+      x.y = e + 1 < V ? row[e + 1] : -INFINITY;
+      x.z = e + 2 < V ? row[e + 2] : -INFINITY;
+      x.w = e + 3 < V ? row[e + 3] : -INFINITY;
+      qq.x = (e < V && residual) ? qrow[e] : 0.f;
+      qq.y = (e + 1 < V && residual) ? qrow[e + 1] : 0.f;
+      qq.z = (e + 2 < V && residual) ? qrow[e + 2] : 0.f;
+      qq.w = (e + 3 < V && residual) ? qrow[e + 3] : 0.f;
+    }
+  };
 
-  // ---- chunk sums of r and p (float-float) ----
-  ff sr = ff_of(0.f), sp = ff_of(0.f);
-  int lr = -1, lp = -1;
-  if (p.vec4) {
-    for (int e = c0 + 4 * tid; e < c1; e += 4 * kAccThreads) {
-      const float4 x = *reinterpret_cast<const float4 *>(row + e);
-      const float4 qv = residual ? __ldcs(reinterpret_cast<const float4 *>(qrow + e))
-                                 : make_float4(0.f, 0.f, 0.f, 0.f);
-      const float xs[4] = {x.x, x.y, x.z, x.w};
-      const float qs[4] = {qv.x, qv.y, qv.z, qv.w};
+  // ---- segment sums of r and p: lane sums of 32 terms added pairwise in
+  // fp32, then a float-float warp sum ----
+  const int sg = c * kAccWarps + warp;
+  if (sg < NS) {
+    float4 xv[8], qv[8];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) load4(sg * kSegTokens + 128 * i + 4 * lane, xv[i], qv[i]);
+    float gr[8], gp[8];
+    int lr = -1, lp = -1;
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      const int e = sg * kSegTokens + 128 * i + 4 * lane;
+      const float xs[4] = {xv[i].x, xv[i].y, xv[i].z, xv[i].w};
+      const float qs[4] = {qv[i].x, qv[i].y, qv[i].z, qv[i].w};
       float rr[4], pz[4];
 #pragma unroll
-      for (int t = 0; t < 4; ++t) {
-        draw_terms(xs[t], qs[t], residual, rs.m, tau, invS, rr[t], pz[t]);
-        if (rr[t] > 0.f) lr = e + t;
-        if (pz[t] > 0.f) lp = e + t;
+      for (int u = 0; u < 4; ++u) {
+        draw_terms(xs[u], qs[u], residual, rs.m, tau, invS, rr[u], pz[u]);
+        lr = rr[u] > 0.f ? e + u : lr;
+        lp = pz[u] > 0.f ? e + u : lp;
       }
-      sr = ff_add(sr, ff_of(sum4(rr[0], rr[1], rr[2], rr[3])));
-      sp = ff_add(sp, ff_of(sum4(pz[0], pz[1], pz[2], pz[3])));
+      gr[i] = sum4(rr[0], rr[1], rr[2], rr[3]);
+      gp[i] = sum4(pz[0], pz[1], pz[2], pz[3]);
     }
-  } else {
-    for (int e = c0 + tid; e < c1; e += kAccThreads) {
-      float rr, pz;
-      draw_terms(row[e], residual ? qrow[e] : 0.f, residual, rs.m, tau, invS, rr, pz);
-      sr = ff_add(sr, ff_of(rr));
-      sp = ff_add(sp, ff_of(pz));
-      if (rr > 0.f) lr = e;
-      if (pz > 0.f) lp = e;
-    }
-  }
-  const ff Sr = block_sum(sr, s_d);
-  const ff Sp = block_sum(sp, s_d);
-  {
-    int v = lr, w = lp;
+    const ff Sr = warp_sum_ff(ff_of(__fadd_rn(__fadd_rn(__fadd_rn(gr[0], gr[1]), __fadd_rn(gr[2], gr[3])),
+                                              __fadd_rn(__fadd_rn(gr[4], gr[5]), __fadd_rn(gr[6], gr[7])))));
+    const ff Sp = warp_sum_ff(ff_of(__fadd_rn(__fadd_rn(__fadd_rn(gp[0], gp[1]), __fadd_rn(gp[2], gp[3])),
+                                              __fadd_rn(__fadd_rn(gp[4], gp[5]), __fadd_rn(gp[6], gp[7])))));
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) {
-      v = max(v, __shfl_xor_sync(0xffffffffu, v, o));
-      w = max(w, __shfl_xor_sync(0xffffffffu, w, o));
+      lr = max(lr, __shfl_xor_sync(0xffffffffu, lr, o));
+      lp = max(lp, __shfl_xor_sync(0xffffffffu, lp, o));
     }
-    if (tid == 0) { s_flag = -1; s_token = -1; }
-    __syncthreads();
-    if ((tid & 31) == 0) { atomicMax(&s_flag, v); atomicMax(&s_token, w); }
-    __syncthreads();
-    if (tid == 0) p.parts[(size_t)b * p.C2 + c] = DrawPart{Sr, Sp, s_flag, s_token, {0, 0}};
+    if (lane == 0) parts[sg] = DrawPart{Sr, Sp, lr, lp, {0, 0}};
   }
 
-  // ---- the last chunk of the sequence draws the token ----
-  __threadfence();
-  __syncthreads();
-  if (tid == 0) s_flag = (atomicAdd(p.draw_tickets + b, 1u) == (unsigned)(p.C2 - 1)) ? 1 : 0;
+  // ---- the last CTA of the sequence draws the token ----
+  __syncthreads();  // every part of this CTA is written
+  if (tid == 0)     // release this CTA's parts, acquire the others'
+    s_flag = atom_add_acq_rel_gpu(p.draw_tickets + b, 1u) == static_cast<unsigned>(p.C2 - 1);
   __syncthreads();
   if (!s_flag) return;
-  __threadfence();
 
-  const DrawPart *parts = p.parts + (size_t)b * p.C2;
   auto part_sum = [&](int cc, bool pmass) -> ff {
-    return pmass ? ff{__ldcg(&parts[cc].sum_p.hi), __ldcg(&parts[cc].sum_p.lo)}
-                 : ff{__ldcg(&parts[cc].sum_r.hi), __ldcg(&parts[cc].sum_r.lo)};
+    const float4 v = __ldcg(reinterpret_cast<const float4 *>(parts + cc));
+    return pmass ? ff{v.z, v.w} : ff{v.x, v.y};
   };
   ff total;
   {
     ff pr = ff_of(0.f);
-    for (int cc = tid; cc < p.C2; cc += kAccThreads) pr = ff_add(pr, part_sum(cc, false));
+    for (int cc = tid; cc < NS; cc += kAccThreads) pr = ff_add(pr, part_sum(cc, false));
     total = block_sum(pr, s_d);
   }
   const bool use_p = !ff_pos(total);  // residual with no mass (rounding only)
   if (use_p) {
     ff pp = ff_of(0.f);
-    for (int cc = tid; cc < p.C2; cc += kAccThreads) pp = ff_add(pp, part_sum(cc, true));
+    for (int cc = tid; cc < NS; cc += kAccThreads) pp = ff_add(pp, part_sum(cc, true));
     total = block_sum(pp, s_d);
   }
   const ff target = ff_mul(total, u_k);
 
-  // chunk holding the target: inclusive float-float scan over chunk sums in order;
-  // chunk cc covers [excl, incl), and excl of cc is bit-identical to incl of
-  // cc - 1, so the intervals tile [0, total) without gaps or overlaps
-  if (tid == 0) { s_chunk = INT_MAX; s_base = ff_of(0.f); }
+  // segment holding the target: inclusive float-float scan over the segment
+  // sums in order; segment cc covers [excl, incl), and excl of cc is
+  // bit-identical to incl of cc - 1, so the intervals tile [0, total)
+  if (tid == 0) { s_seg = INT_MAX; s_base = ff_of(0.f); }
   ff carry = ff_of(0.f);
-  for (int base = 0; base < p.C2; base += kAccThreads) {
+  for (int base = 0; base < NS; base += kAccThreads) {
     const int cc = base + tid;
-    const ff v = cc < p.C2 ? part_sum(cc, use_p) : ff_of(0.f);
+    const ff v = cc < NS ? part_sum(cc, use_p) : ff_of(0.f);
     ff excl_local, blk_total;
     const ff incl_local = block_inclusive_scan(v, s_scan, &excl_local, &blk_total);
     const ff excl = ff_add(carry, excl_local), incl = ff_add(carry, incl_local);
-    if (cc < p.C2 && ff_pos(v) && ff_lt(target, incl) && !ff_lt(target, excl))
-      atomicMin(&s_chunk, cc);
+    if (cc < NS && ff_pos(v) && ff_lt(target, incl) && !ff_lt(target, excl)) atomicMin(&s_seg, cc);
     __syncthreads();
-    if (s_chunk == cc) s_base = excl;
+    if (s_seg == cc) s_base = excl;
     carry = ff_add(carry, blk_total);
     __syncthreads();
-    if (s_chunk != INT_MAX) break;
+    if (s_seg != INT_MAX) break;
   }
   __syncthreads();
   int token = -1;
-  if (s_chunk == INT_MAX) {
+  if (s_seg == INT_MAX) {
     // u*S at or past the total (rounding): the last token with positive mass
     int last = -1;
-    for (int cc = tid; cc < p.C2; cc += kAccThreads)
+    for (int cc = tid; cc < NS; cc += kAccThreads)
       last = max(last, use_p ? __ldcg(&parts[cc].last_p) : __ldcg(&parts[cc].last_r));
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) last = max(last, __shfl_xor_sync(0xffffffffu, last, o));
-    if (tid == 0) s_last = -1;
+    if (tid == 0) s_token = -1;
     __syncthreads();
-    if ((tid & 31) == 0) atomicMax(&s_last, last);
+    if (lane == 0) atomicMax(&s_token, last);
     __syncthreads();
-    token = s_last;
+    token = s_token;
   } else {
-    // scan the chunk in ascending token order: thread t owns a contiguous run
-    const int cc = s_chunk;
-    const int e0 = cc * p.CV2, e1 = min(V, e0 + p.CV2);
-    const int len = e1 - e0;
-    for (int e = tid; e < len; e += kAccThreads) {
-      float rr, pz;
-      draw_terms(row[e0 + e], residual ? qrow[e0 + e] : 0.f, residual, rs.m, tau, invS, rr, pz);
-      s_r[e] = use_p ? pz : rr;
-    }
-    __syncthreads();
-    const int per = (len + kAccThreads - 1) / kAccThreads;
-    const int a0 = tid * per, a1 = min(len, a0 + per);
+    // the segment in ascending token order: thread t owns tokens 4t .. 4t+3
+    // (terms recomputed exactly as in the segment sums)
+    const int cc = s_seg;
+    const int e = cc * kSegTokens + 4 * tid;
+    float4 xv, qv;
+    load4(e, xv, qv);
+    const float xs[4] = {xv.x, xv.y, xv.z, xv.w};
+    const float qs[4] = {qv.x, qv.y, qv.z, qv.w};
+    float t[4];
     ff mine = ff_of(0.f);
-    for (int e = a0; e < a1; ++e) mine = ff_add(mine, ff_of(s_r[e]));
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      float rr, pz;
+      draw_terms(xs[u], qs[u], residual, rs.m, tau, invS, rr, pz);
+      t[u] = use_p ? pz : rr;
+      mine = ff_add(mine, ff_of(t[u]));
+    }
     ff excl, unused;
     block_inclusive_scan(mine, s_scan, &excl, &unused);
     ff cum = ff_add(s_base, excl);
     if (tid == 0) s_token = INT_MAX;
     __syncthreads();
-    for (int e = a0; e < a1; ++e) {
-      cum = ff_add(cum, ff_of(s_r[e]));
-      if (ff_lt(target, cum)) { atomicMin(&s_token, e0 + e); break; }
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      cum = ff_add(cum, ff_of(t[u]));
+      if (t[u] > 0.f && ff_lt(target, cum)) {
+        atomicMin(&s_token, e + u);
+        break;
+      }
     }
     __syncthreads();
     token = s_token;
     if (token == INT_MAX) {
-      // rounding put the target past this chunk's own sum: its last positive token
+      // rounding put the target past the segment's own running sum: its last
+      // positive token
       token = use_p ? __ldcg(&parts[cc].last_p) : __ldcg(&parts[cc].last_r);
     }
   }
@@ -867,39 +716,301 @@ accept_draw_kernel(const __grid_constant__ AccParams p) {
   }
 }
 
+
+__global__ void __launch_bounds__(kAccThreads, 3)
+accept_draw_kernel(const __grid_constant__ AccParams p) {
+  // The previous kernel (the decision kernel of this call) lets this grid
+  // start only after it has itself waited for the kernel before the call, so
+  // the call's inputs (temperature, uniforms) are in place already; j and
+  // the row statistics are waited for.
+  grid_launch_dependents();
+  const int c = blockIdx.x, b = blockIdx.y;
+  const int k = p.k;
+  const float tau = p.tau[b];
+  if (!(tau > 0.0f)) return;  // greedy sequences are complete
+  const float u_k = p.u[(size_t)b * (k + 1) + k];
+  grid_dependency_wait();     // j and the row statistics come from the previous kernel
+  const int j = __ldcg(&p.seqs[b].j);
+  const RowStat rs = {__ldcg(&p.rows[(size_t)b * (k + 1) + j].m),
+                      __ldcg(&p.rows[(size_t)b * (k + 1) + j].arg),
+                      ff{__ldcg(&p.rows[(size_t)b * (k + 1) + j].S.hi),
+                         __ldcg(&p.rows[(size_t)b * (k + 1) + j].S.lo)}};
+  draw_residual(p, b, c, j, rs, tau, u_k);
+}
+
+// --------------------------------------------------------------------------
+// Two-kernel acceptance for vocabularies beyond one cluster (V > 16 x 2048).
+//
+// accept_chunks_kernel streams the (k+1) x V logits of every sequence once.
+// The B (k+1) rows are cut into 1024-token segments ("chunks"), numbered row
+// by row, and warp g of NW1 owns chunks [g U / NW1, (g+1) U / NW1) of the U
+// in all: a few consecutive chunks, at most two or three rows.  Lane l reads
+// tokens 128 i + 4 l .. +3 of a chunk (eight 16-byte loads), and the next
+// chunk's loads are in flight while the current one is folded into per-lane
+// running state (max, first index, float-float sum of exp((x - max)/tau)).
+// At the end of each run of chunks of one row the warp combines its lanes
+// and writes one run record; the runs of row R are stored in warp order, so
+// that run t of the row is the one of warp warp_of(R C1) + t.
+//
+// accept_finish_kernel, grid (C2, B): every CTA of sequence b combines the
+// run records of the k+1 rows (one warp per row, in run order), reads the
+// draft tokens' logits and probabilities, takes the k decisions (the same
+// device function as the other paths; CTA 0 writes the outputs) and, for a
+// sampled sequence, does its part of the residual draw (draw_residual).
+// --------------------------------------------------------------------------
+
+// The warp of the chunk kernel owning chunk u: the largest g with
+// floor(g U / NW) <= u (warps with empty ranges are never returned).
+__device__ __forceinline__ int warp_of(int u, int U, int NW) {
+  return static_cast<int>(((long long)(u + 1) * NW - 1) / U);
+}
+
+// The 32 tokens of lane `lane` in chunk c of a row: c*1024 + 128 i + 4 lane + t
+// (tokens at or past V read as -inf).
+__device__ __forceinline__ void load_chunk(const AccParams &p, int row, int c, int lane,
+                                           float4 (&x)[8]) {
+  const float *rp = p.logits + (size_t)row * p.V;
+#pragma unroll
+  for (int i = 0; i < 8; ++i) {
+    const int e = c * kSegTokens + 128 * i + 4 * lane;
+    if (p.vec4) {
+      x[i] = e < p.V ? __ldcg(reinterpret_cast<const float4 *>(rp + e))
+                     : make_float4(-INFINITY, -INFINITY, -INFINITY, -INFINITY);
+    } else {
+      x[i].x = e < p.V ? __ldcg(rp + e) : -INFINITY;
+      x[i].y = e + 1 < p.V ? __ldcg(rp + e + 1) : -INFINITY;
+      x[i].z = e + 2 < p.V ? __ldcg(rp + e + 2) : -INFINITY;
+      x[i].w = e + 3 < p.V ? __ldcg(rp + e + 3) : -INFINITY;
+    }
+  }
+}
+
+// State of one warp over its current run (consecutive chunks of one row).
+// Each lane keeps the max of its own tokens so far, the first index holding
+// it and the float-float sum of exp((x - max)/tau) over them; the warp
+// combines the lanes once, at the end of the run.
+struct RunState {
+  int row, c, start_chunk, len;
+  float tau, scale;  // scale = log2(e) / tau, rounded once
+  bool greedy;
+  float lm;          // lane max
+  int li;            // its first index
+  ff lS;             // lane sum, relative to lm
+};
+
+__device__ __forceinline__ void run_begin(const AccParams &p, RunState &st, int row, int c) {
+  st.row = row;
+  st.c = c;
+  st.start_chunk = c;
+  st.len = 0;
+  st.tau = __ldg(p.tau + row / (p.k + 1));
+  st.greedy = !(st.tau > 0.0f);
+  st.scale = st.greedy ? 0.f : __fdiv_rn(1.44269504088896341f, st.tau);
+  st.lm = -INFINITY;
+  st.li = INT_MAX;
+  st.lS = ff_of(0.f);
+}
+
+// Folds chunk st.c (its tokens in x) into the lane state.
+__device__ __forceinline__ void run_chunk(RunState &st, int lane, const float4 (&x)[8]) {
+  float cm = -INFINITY;
+#pragma unroll
+  for (int i = 0; i < 8; ++i) cm = fmaxf(cm, fmaxf(fmaxf(x[i].x, x[i].y), fmaxf(x[i].z, x[i].w)));
+  if (st.len == 0 || cm > st.lm) {
+    // new lane max (or the run's first chunk): its first index in this chunk,
+    // and the sum so far moved to the new reference
+    int fi = INT_MAX;
+#pragma unroll
+    for (int i = 7; i >= 0; --i) {  // descending, so the first match wins
+      const int e = st.c * kSegTokens + 128 * i + 4 * lane;
+      fi = x[i].w == cm ? e + 3 : fi;
+      fi = x[i].z == cm ? e + 2 : fi;
+      fi = x[i].y == cm ? e + 1 : fi;
+      fi = x[i].x == cm ? e : fi;
+    }
+    if (ff_pos(st.lS)) st.lS = ff_mul(st.lS, exp_diff_accurate(st.lm, cm, st.tau));
+    st.lm = cm;
+    st.li = fi;
+  }
+  if (!st.greedy && st.lm != -INFINITY) {
+    // 2^((x - lm) log2(e)/tau): the difference and the product each rounded
+    // once per token (a term's relative error grows with |x - lm| x 1e-7
+    // with no common bias), 2^ by the hardware approximation; the 32 terms
+    // are added pairwise in fp32 before one float-float add
+    float t[8];
+#pragma unroll
+    for (int i = 0; i < 8; ++i)
+      t[i] = sum4(ex2_approx(__fmul_rn(__fsub_rn(x[i].x, st.lm), st.scale)),
+                  ex2_approx(__fmul_rn(__fsub_rn(x[i].y, st.lm), st.scale)),
+                  ex2_approx(__fmul_rn(__fsub_rn(x[i].z, st.lm), st.scale)),
+                  ex2_approx(__fmul_rn(__fsub_rn(x[i].w, st.lm), st.scale)));
+    st.lS = ff_add(st.lS, ff_of(__fadd_rn(__fadd_rn(__fadd_rn(t[0], t[1]), __fadd_rn(t[2], t[3])),
+                                          __fadd_rn(__fadd_rn(t[4], t[5]), __fadd_rn(t[6], t[7])))));
+  }
+  ++st.len;
+}
+
+// Ends the warp's run: combines the lanes and writes the run's record.
+__device__ __forceinline__ void run_end(const AccParams &p, const RunState &st, int lane, int gw,
+                                        int U) {
+  float wm = st.lm;
+  int wi = st.li;
+  warp_argmax(wm, wi);
+  ff S = ff_of(0.f);
+  if (!st.greedy && wm != -INFINITY) {
+    ff mine = ff_of(0.f);
+    if (ff_pos(st.lS)) mine = ff_mul(st.lS, exp_diff_accurate(st.lm, wm, st.tau));
+    S = warp_sum_ff(mine);
+  }
+  if (lane == 0) {
+    const int CPR = p.C1;
+    const int t = gw - warp_of(st.row * CPR, U, p.NW1);  // the run's place in its row
+    p.runs[(size_t)st.row * CPR + t] = RowStat{wm, wi, S};
+  }
+}
+
+__global__ void __launch_bounds__(kAccThreads, 2)
+accept_chunks_kernel(const __grid_constant__ AccParams p) {
+  // Every input may come from the previous kernel on the stream: wait for
+  // it before reading anything, and only then let the finishing kernel be
+  // scheduled (so that it too starts after that kernel completed).
+  grid_dependency_wait();
+  grid_launch_dependents();
+  const int lane = threadIdx.x & 31;
+  const int gw = blockIdx.x * kAccWarps + (threadIdx.x >> 5);
+  const int CPR = p.C1;
+  const int U = p.B * (p.k + 1) * CPR;  // < 2^31: the host checks V * (k + 1) and B
+  const int u0 = static_cast<int>((long long)gw * U / p.NW1);
+  const int u1 = static_cast<int>((long long)(gw + 1) * U / p.NW1);
+  if (u0 >= u1) return;
+  RunState st;
+  run_begin(p, st, u0 / CPR, u0 % CPR);
+  // two register buffers: chunk u + 1 is loading while chunk u is reduced
+  float4 xa[8], xb[8];
+  load_chunk(p, st.row, st.c, lane, xa);
+  auto step = [&](int u, const float4 (&cur)[8], float4 (&nxt)[8]) {
+    int nrow = st.row, nc = st.c + 1;
+    if (nc == CPR) { nc = 0; ++nrow; }
+    if (u + 1 < u1) load_chunk(p, nrow, nc, lane, nxt);
+    run_chunk(st, lane, cur);
+    if (nc == 0 || u + 1 == u1) {
+      run_end(p, st, lane, gw, U);
+      if (u + 1 < u1) run_begin(p, st, nrow, 0);
+    } else {
+      st.c = nc;
+    }
+  };
+  for (int u = u0; u < u1; u += 2) {
+    step(u, xa, xb);
+    if (u + 1 < u1) step(u + 1, xb, xa);
+  }
+}
+
+// Combines the run records of target row `row` (in run order, which is
+// chunk order) into the row's max, first argmax and float-float sum rescaled
+// to the max.  Executed by one whole warp; all loads are issued before any
+// is used.
+__device__ __forceinline__ RowStat combine_runs(const AccParams &p, int row, float tau,
+                                                bool greedy) {
+  constexpr int kPer = 4;  // records per lane and pass
+  const int lane = threadIdx.x & 31, CPR = p.C1;
+  const int U = p.B * (p.k + 1) * CPR;
+  const int g0 = warp_of(row * CPR, U, p.NW1);
+  const int n = warp_of(row * CPR + CPR - 1, U, p.NW1) - g0 + 1;
+  const float4 *rr = reinterpret_cast<const float4 *>(p.runs + (size_t)row * CPR);
+  float mv = -INFINITY;
+  int mi = INT_MAX;
+  ff Sr = ff_of(0.f);
+  for (int base = 0; base < n; base += 32 * kPer) {  // one pass unless n > 128
+    float4 a[kPer];
+#pragma unroll
+    for (int t = 0; t < kPer; ++t) {
+      const int i = base + lane + 32 * t;
+      a[t] = i < n ? __ldcg(rr + i) : make_float4(-INFINITY, __int_as_float(INT_MAX), 0.f, 0.f);
+    }
+    float bm = -INFINITY;
+    int bi = INT_MAX;
+#pragma unroll
+    for (int t = 0; t < kPer; ++t)
+      if (better(a[t].x, __float_as_int(a[t].y), bm, bi)) { bm = a[t].x; bi = __float_as_int(a[t].y); }
+    warp_argmax(bm, bi);
+    if (!greedy) {
+      // the pass's sums relative to its max, then the running sum moved to
+      // the larger of the two maxima
+      ff ps = ff_of(0.f);
+#pragma unroll
+      for (int t = 0; t < kPer; ++t) {
+        const ff cS = ff{a[t].z, a[t].w};
+        if (ff_pos(cS)) ps = ff_add(ps, ff_mul(cS, exp_diff_accurate(a[t].x, bm, tau)));
+      }
+      ps = warp_sum_ff(ps);
+      if (bm > mv) {
+        if (ff_pos(Sr)) Sr = ff_mul(Sr, exp_diff_accurate(mv, bm, tau));
+        Sr = ff_add(Sr, ps);
+      } else if (ff_pos(ps)) {
+        Sr = ff_add(Sr, ff_mul(ps, exp_diff_accurate(bm, mv, tau)));
+      }
+    }
+    if (better(bm, bi, mv, mi)) { mv = bm; mi = bi; }
+  }
+  return RowStat{mv, mi, Sr};
+}
+
+__global__ void __launch_bounds__(kAccThreads, 3)
+accept_finish_kernel(const __grid_constant__ AccParams p) {
+  __shared__ int s_acc[SF_MAX_DRAFT], s_j;
+  __shared__ float s_rm[SF_MAX_DRAFT + 1], s_rlx[SF_MAX_DRAFT + 1], s_rqx[SF_MAX_DRAFT + 1];
+  __shared__ int s_rarg[SF_MAX_DRAFT + 1], s_rhx[SF_MAX_DRAFT + 1];
+  __shared__ ff s_rS[SF_MAX_DRAFT + 1];
+  const int c = blockIdx.x, b = blockIdx.y, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int k = p.k, V = p.V;
+  grid_dependency_wait();  // the run records (and every input) follow the previous kernel
+  grid_launch_dependents();
+  const float tau = p.tau[b];
+  const bool greedy = !(tau > 0.0f);
+  int my_tok = -1;
+  float my_u = 0.f;
+  if (tid < k) {
+    // draft token i's logit and draft probability, read directly
+    my_tok = p.tokens[(size_t)b * k + tid];
+    my_u = p.u[(size_t)b * (k + 1) + tid];
+    const bool ok = my_tok >= 0 && my_tok < V;
+    s_rlx[tid] = ok ? p.logits[((size_t)b * (k + 1) + tid) * V + my_tok] : 0.f;
+    s_rqx[tid] = ok ? p.q[((size_t)b * k + tid) * V + my_tok] : 0.f;
+    s_rhx[tid] = ok ? 1 : 0;
+  }
+  for (int r = warp; r <= k; r += kAccWarps) {
+    const RowStat rs = combine_runs(p, b * (k + 1) + r, tau, greedy);
+    if (lane == 0) {
+      s_rm[r] = rs.m;
+      s_rarg[r] = rs.arg;
+      s_rS[r] = rs.S;
+    }
+  }
+  __syncthreads();
+  decide_sequence(p, b, greedy, tau, my_tok, my_u, s_rm, s_rarg, s_rS, s_rlx, s_rqx, s_rhx, s_acc,
+                  c == 0, &s_j);
+  __syncthreads();
+  if (greedy) return;  // CTA 0 wrote the argmax of row j
+  const int j = s_j;
+  const float u_k = p.u[(size_t)b * (k + 1) + k];
+  draw_residual(p, b, c, j, RowStat{s_rm[j], s_rarg[j], s_rS[j]}, tau, u_k);
+}
+
 // --------------------------------------------------------------------------
 // host side
 // --------------------------------------------------------------------------
 struct AccPlan {
-  int C1, CV1, C2, CV2;
+  int C1, C2;  // segments per row, draw CTAs per row
 };
 
 struct AccLayout {
-  size_t seq_tickets, draw_tickets, chunks, rows, seqs, parts, total;
+  size_t draw_tickets, runs, rows, seqs, parts, total;
 };
 
-static int chunking(long long target_ctas, int V, int rows, int *C, int *CV) {
-  const long long min_chunks = (V + kMaxChunk - 1) / kMaxChunk;
-  const long long max_chunks = V > 1024 ? (V + 1023) / 1024 : 1;
-  long long want = (target_ctas + rows - 1) / rows;
-  if (want < min_chunks) want = min_chunks;
-  if (want > max_chunks) want = max_chunks;
-  if (want < 1) want = 1;
-  long long cv = (V + want - 1) / want;
-  cv = (cv + 3) / 4 * 4;
-  if (cv > kMaxChunk) cv = kMaxChunk;
-  *CV = static_cast<int>(cv);
-  *C = static_cast<int>((V + cv - 1) / cv);
-  return SF_OK;
-}
-
-static int plan_accept(int B, int k, int V, AccPlan *plan) {
-  DeviceInfo dev;
-  int st = current_device(&dev);
-  if (st != SF_OK) return st;
-  const long long target = 4LL * dev.sm_count;  // ~ 4 CTAs of 256 threads per SM
-  chunking(target, V, B * (k + 1), &plan->C1, &plan->CV1);
-  chunking(target, V, B, &plan->C2, &plan->CV2);
+static int plan_accept(int V, AccPlan *plan) {
+  plan->C1 = (V + kSegTokens - 1) / kSegTokens;
+  plan->C2 = (plan->C1 + kAccWarps - 1) / kAccWarps;
   return SF_OK;
 }
 
@@ -907,12 +1018,11 @@ static AccLayout acc_layout(int B, int k, const AccPlan &pl) {
   AccLayout l;
   const size_t R = (size_t)B * (k + 1);
   size_t off = 256;
-  l.seq_tickets = off; off = round_up(off + 4 * (size_t)B, 256);
   l.draw_tickets = off; off = round_up(off + 4 * (size_t)B, 256);
-  l.chunks = off; off = round_up(off + sizeof(ChunkRec) * R * pl.C1, 256);
+  l.runs = off; off = round_up(off + sizeof(RowStat) * R * pl.C1, 256);
   l.rows = off; off = round_up(off + sizeof(RowStat) * R, 256);
   l.seqs = off; off = round_up(off + sizeof(SeqState) * (size_t)B, 256);
-  l.parts = off; off = round_up(off + sizeof(DrawPart) * (size_t)B * pl.C2, 256);
+  l.parts = off; off = round_up(off + sizeof(DrawPart) * (size_t)B * pl.C1, 256);
   l.total = off;
   return l;
 }
@@ -986,7 +1096,7 @@ extern "C" {
 size_t sf_accept_workspace_size(int B, int k, int V) {
   if (sf::check_accept_shapes(B, k, V) != SF_OK) return 0;
   sf::AccPlan plan;
-  if (sf::plan_accept(B, k, V, &plan) != SF_OK) return 0;
+  if (sf::plan_accept(V, &plan) != SF_OK) return 0;
   return sf::acc_layout(B, k, plan).total;
 }
 
@@ -1018,7 +1128,7 @@ int sf_accept(const float *target_logits, const float *draft_probs,
   if (!workspace || !aligned(workspace, 256))
     return fail(SF_ERR_WORKSPACE, "workspace must be non-NULL and 256-byte aligned");
   AccPlan plan;
-  st = plan_accept(B, k, V, &plan);
+  st = plan_accept(V, &plan);
   if (st != SF_OK) return st;
   const AccLayout lay = acc_layout(B, k, plan);
   if (workspace_bytes < lay.total)
@@ -1035,9 +1145,8 @@ int sf_accept(const float *target_logits, const float *draft_probs,
   prm.out_tokens = out_tokens;
   prm.ratio = accept_ratio;
   prm.status = reinterpret_cast<uint32_t *>(ws);
-  prm.seq_tickets = reinterpret_cast<uint32_t *>(ws + lay.seq_tickets);
   prm.draw_tickets = reinterpret_cast<uint32_t *>(ws + lay.draw_tickets);
-  prm.chunks = reinterpret_cast<ChunkRec *>(ws + lay.chunks);
+  prm.runs = reinterpret_cast<RowStat *>(ws + lay.runs);
   prm.rows = reinterpret_cast<RowStat *>(ws + lay.rows);
   prm.seqs = reinterpret_cast<SeqState *>(ws + lay.seqs);
   prm.parts = reinterpret_cast<DrawPart *>(ws + lay.parts);
@@ -1045,9 +1154,8 @@ int sf_accept(const float *target_logits, const float *draft_probs,
   prm.k = k;
   prm.V = V;
   prm.C1 = plan.C1;
-  prm.CV1 = plan.CV1;
   prm.C2 = plan.C2;
-  prm.CV2 = plan.CV2;
+  prm.NW1 = 0;
   prm.vec4 = (V % 4 == 0) && aligned(target_logits, 16) && aligned(draft_probs, 16);
 
   // One cluster per sequence when a row fits 16 slices: a single launch
@@ -1083,18 +1191,25 @@ int sf_accept(const float *target_logits, const float *draft_probs,
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
   attr[0].val.programmaticStreamSerializationAllowed = 1;
+  DeviceInfo dev;
+  st = current_device(&dev);
+  if (st != SF_OK) return st;
+  const long long units = (long long)B * (k + 1) * plan.C1;
+  long long ctas = (units + kAccWarps - 1) / kAccWarps;
+  if (ctas > 2LL * dev.sm_count) ctas = 2LL * dev.sm_count;  // two CTAs per SM
+  prm.NW1 = static_cast<int>(ctas) * kAccWarps;
   cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(plan.C1, k + 1, B);
+  cfg.gridDim = dim3(static_cast<unsigned>(ctas));
   cfg.blockDim = dim3(kAccThreads);
   cfg.dynamicSmemBytes = 0;
   cfg.stream = stream;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  cudaError_t e = cudaLaunchKernelEx(&cfg, accept_stats_kernel, prm);
-  if (e != cudaSuccess) return fail(SF_ERR_CUDA, "accept stats launch: %s", cudaGetErrorString(e));
+  cudaError_t e = cudaLaunchKernelEx(&cfg, accept_chunks_kernel, prm);
+  if (e != cudaSuccess) return fail(SF_ERR_CUDA, "accept chunks launch: %s", cudaGetErrorString(e));
   cfg.gridDim = dim3(plan.C2, B);
-  e = cudaLaunchKernelEx(&cfg, accept_draw_kernel, prm);
-  if (e != cudaSuccess) return fail(SF_ERR_CUDA, "accept draw launch: %s", cudaGetErrorString(e));
+  e = cudaLaunchKernelEx(&cfg, accept_finish_kernel, prm);
+  if (e != cudaSuccess) return fail(SF_ERR_CUDA, "accept finish launch: %s", cudaGetErrorString(e));
   return SF_OK;
 }
 
@@ -1102,7 +1217,7 @@ size_t sf_verify_lm_head_accept_workspace_size(int B, int k, int V) {
   using namespace sf;
   if (check_accept_shapes(B, k, V) != SF_OK || B * (k + 1) > SF_MAX_DRAFT_ROWS) return 0;
   AccPlan plan;
-  if (plan_accept(B, k, V, &plan) != SF_OK) return 0;
+  if (plan_accept(V, &plan) != SF_OK) return 0;
   DeviceInfo dev;
   if (current_device(&dev) != SF_OK) return 0;
   const size_t G = static_cast<size_t>(projection_groups(V, dev.sm_count));
@@ -1129,7 +1244,7 @@ int sf_verify_lm_head_accept(const void *hidden, const void *weight, const float
   if (!workspace || !aligned(workspace, 256))
     return fail(SF_ERR_WORKSPACE, "workspace must be non-NULL and 256-byte aligned");
   AccPlan plan;
-  st = plan_accept(B, k, V, &plan);
+  st = plan_accept(V, &plan);
   if (st != SF_OK) return st;
   DeviceInfo dev;
   st = current_device(&dev);
@@ -1159,9 +1274,8 @@ int sf_verify_lm_head_accept(const void *hidden, const void *weight, const float
   prm.out_tokens = out_tokens;
   prm.ratio = accept_ratio;
   prm.status = reinterpret_cast<uint32_t *>(ws);
-  prm.seq_tickets = reinterpret_cast<uint32_t *>(ws + lay.seq_tickets);
   prm.draw_tickets = reinterpret_cast<uint32_t *>(ws + lay.draw_tickets);
-  prm.chunks = reinterpret_cast<ChunkRec *>(ws + lay.chunks);
+  prm.runs = reinterpret_cast<RowStat *>(ws + lay.runs);
   prm.rows = reinterpret_cast<RowStat *>(ws + lay.rows);
   prm.seqs = reinterpret_cast<SeqState *>(ws + lay.seqs);
   prm.parts = reinterpret_cast<DrawPart *>(ws + lay.parts);
@@ -1169,9 +1283,8 @@ int sf_verify_lm_head_accept(const void *hidden, const void *weight, const float
   prm.k = k;
   prm.V = V;
   prm.C1 = plan.C1;
-  prm.CV1 = plan.CV1;
   prm.C2 = plan.C2;
-  prm.CV2 = plan.CV2;
+  prm.NW1 = 0;
   prm.vec4 = (V % 4 == 0) && aligned(logits, 16) && aligned(draft_probs, 16);
 
   cudaLaunchAttribute attr[1];

@@ -166,10 +166,21 @@ def test_equal_distributions_accept_all_and_use_the_bonus_row(oracle_mod):
     assert (n == k).all()
 
 
-def test_temperatures_other_than_one(oracle_mod):
-    inp = make_accept_case(128, 4, 32000, seed=7)
-    inp.temperature = np.where(np.arange(128) % 3 == 0, 0.7, 1.3).astype(np.float32)
+@pytest.mark.parametrize("V", [32000, 152064])
+def test_temperatures_other_than_one(oracle_mod, V):
+    B = 128 if V < 100000 else 24
+    inp = make_accept_case(B, 4, V, seed=7)
+    inp.temperature = np.where(np.arange(B) % 3 == 0, 0.7, 1.3).astype(np.float32)
     _check(oracle_mod, inp)
+
+
+def test_warp_runs_longer_than_32_chunks(oracle_mod):
+    # 40 x 17 rows of 149 chunks: on a 152-SM part every warp of the chunk
+    # kernel folds ~42 consecutive chunks, so runs cross rows mid-warp and
+    # span more chunk records than a warp has lanes
+    # (17 decisions per sequence: more of them fall within the oracle's margin)
+    inp = make_accept_case(40, 16, 152064, seed=40, mode="alternate")
+    _check(oracle_mod, inp, max_excluded_frac=0.1)
 
 
 def test_out_of_range_draft_token_is_flagged_and_rejected(oracle_mod):
@@ -195,7 +206,7 @@ def test_repeated_calls_are_bit_identical():
 
 def test_kernel_launch_counts_follow_the_vocabulary():
     # one cluster kernel while a row fits 16 slices of 2048 tokens, else the
-    # statistics and draw kernels
+    # chunk and finish kernels
     assert sfv.accept_kernel_launches(1, 5, 32000) == 1
     assert sfv.accept_kernel_launches(4, 8, 32768) == 1
     assert sfv.accept_kernel_launches(4, 8, 32769) == 2
