@@ -71,6 +71,7 @@ __device__ void tile_prefix(const AttnParams &p, int *s_prefix, int *s_len, int 
   const int per = (p.B + NT - 1) / NT;
   const int b0 = tid * per;
   int local = 0;
+#pragma unroll 1
   for (int b = b0; b < b0 + per && b < p.B; ++b) {
     int T = p.seq_lens[b];
     if (T < p.n_q || T > p.max_tokens) {
@@ -89,8 +90,10 @@ __device__ void tile_prefix(const AttnParams &p, int *s_prefix, int *s_len, int 
   if (lane == 31) s_warp[warp] = incl;
   __syncthreads();
   int warp_off = 0;
+#pragma unroll 1
   for (int w = 0; w < warp; ++w) warp_off += s_warp[w];
   int run = warp_off + incl - local;
+#pragma unroll 1
   for (int b = b0; b < b0 + per && b < p.B; ++b) {
     s_prefix[b] = run;
     run += (s_len[b] + kTileTokens - 1) / kTileTokens;
@@ -135,6 +138,7 @@ __device__ void aligned_prefix(const AttnParams &p, const int *s_prefix, int Ta,
   const int per = (p.B + NT - 1) / NT;
   const int b0 = tid * per;
   int local = 0;
+#pragma unroll 1
   for (int b = b0; b < b0 + per && b < p.B; ++b)
     local += p.H_kv * ((s_prefix[b + 1] - s_prefix[b] + Ta - 1) / Ta);
   int incl = local;
@@ -146,8 +150,10 @@ __device__ void aligned_prefix(const AttnParams &p, const int *s_prefix, int Ta,
   if (lane == 31) s_warp[warp] = incl;
   __syncthreads();
   int warp_off = 0;
+#pragma unroll 1
   for (int w = 0; w < warp; ++w) warp_off += s_warp[w];
   int run = warp_off + incl - local;
+#pragma unroll 1
   for (int b = b0; b < b0 + per && b < p.B; ++b) {
     s_out[b] = run;
     run += p.H_kv * ((s_prefix[b + 1] - s_prefix[b] + Ta - 1) / Ta);

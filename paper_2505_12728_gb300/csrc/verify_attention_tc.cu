@@ -169,14 +169,17 @@ __device__ TcPartition tc_partition(const AttnParams &p, const int *s_prefix, in
     tp.aligned = Ta <= Tmin + kAlignSlackTiles;
     // the smallest piece length whose pieces still fit the grid (Ta always
     // does: each segment's ceiling adds less than one CTA)
+#pragma unroll 1
     for (int cand = Tmin; tp.aligned && cand < Ta; ++cand) {
       int local = 0;
+#pragma unroll 1
       for (int b = tid; b < p.B; b += NT) local += (s_prefix[b + 1] - s_prefix[b] + cand - 1) / cand;
 #pragma unroll
       for (int o = 16; o > 0; o >>= 1) local += __shfl_xor_sync(0xffffffffu, local, o);
       if (lane == 0) s_scratch[warp] = local;
       __syncthreads();
       int need = 0;
+#pragma unroll 1
       for (int w = 0; w < NT / 32; ++w) need += s_scratch[w];
       __syncthreads();
       if (static_cast<long long>(need) * p.H_kv <= p.G) {
@@ -833,15 +836,19 @@ verify_tc_merge_kernel(const __grid_constant__ AttnParams p) {
   __syncthreads();
   const TcPartition tp = tc_partition<kTcMergeThreads>(p, s_prefix, s_cpre, s_scratch + 8);
   grid_dependency_wait();
+  // work units of kTcMergeThreads items of one segment (32-bit indices:
+  // the units of all segments number fewer than 2^31)
   const int per_seg = p.R * C4;
-  const long long total = (long long)per_seg * p.B * p.H_kv;
+  const int units_per_seg = (per_seg + kTcMergeThreads - 1) / kTcMergeThreads;
+  const int units = p.B * p.H_kv * units_per_seg;
   const size_t stride = (size_t)p.slot_stride;
-  for (long long item = (long long)blockIdx.x * kTcMergeThreads + threadIdx.x; item < total;
-       item += (long long)gridDim.x * kTcMergeThreads) {
-    const int seg = static_cast<int>(item / per_seg);
-    const int rem = static_cast<int>(item % per_seg);
-    const int c4 = rem / p.R, r = rem % p.R;
-    const int b = seg / p.H_kv, h_kv = seg % p.H_kv;
+#pragma unroll 1
+  for (int unit = blockIdx.x; unit < units; unit += gridDim.x) {
+    const int seg = unit / units_per_seg;
+    const int rem = (unit - seg * units_per_seg) * kTcMergeThreads + threadIdx.x;
+    if (rem >= per_seg) continue;
+    const int c4 = rem / p.R, r = rem - c4 * p.R;
+    const int b = seg / p.H_kv, h_kv = seg - b * p.H_kv;
     int c_first, n_pieces;
     tc_segment(tp, p, s_prefix, s_cpre, b, h_kv, c_first, n_pieces);
     if (n_pieces <= 1) continue;  // the split kernel wrote the output

@@ -246,6 +246,26 @@ def test_kernel_launch_counts_follow_the_rows_per_kv_head():
     assert sfv.verify_attention_kernel_launches(16, 8, 28, 4, 128, 2049) == 2
 
 
+@pytest.mark.parametrize("B,n_q,H_q,H_kv,d,prefix_range", [
+    (1, 16, 8, 1, 128, (20000, 20000)),  # one 128-row segment over every CTA
+    (1, 16, 8, 1, 64, (20000, 20000)),
+    (1, 8, 28, 4, 128, (30000, 30000)),  # four 56-row segments of ~38 pieces each
+    (40, 8, 28, 4, 128, (500, 3000)),    # 160 segments > 152 CTAs: balanced partition,
+                                         # a CTA's first and last pieces split
+])
+def test_tcgen05_many_piece_merges_match_oracle(oracle_mod, B, n_q, H_q, H_kv, d, prefix_range):
+    # Segments split over many CTAs (up to every CTA of the grid, 128 rows)
+    # and CTAs holding pieces of several segments: the merge kernel combines
+    # the partials of all pieces of each split segment, in batches.
+    rng = np.random.default_rng(4000 + B + d)
+    prefixes = [int(x) for x in rng.integers(prefix_range[0], prefix_range[1] + 1, size=B)]
+    case = make_attention_case(B, n_q, H_q, H_kv, d, prefixes, seed=4100 + B + d)
+    ref_out, ref_lse = oracle_attention(oracle_mod, case)
+    for splits in (0, 37):
+        out, lse = run_attention(case, num_splits=splits)
+        assert_attention_close(out, lse, ref_out, ref_lse)
+
+
 @pytest.mark.parametrize("n_q,H_q,H_kv,d", [
     (4, 8, 8, 64),      # mma.sync kernel: 8192 segments of one or two tiles
     (8, 28, 4, 128),    # tcgen05 kernel: 56 rows per KV head, 4096 segments
