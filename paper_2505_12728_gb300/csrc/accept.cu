@@ -869,15 +869,28 @@ __device__ __forceinline__ void run_end(const AccParams &p, const RunState &st, 
   }
 }
 
+// Chunk ring of the bulk-copy path: kChunkStages 4 KB stages per warp (the
+// chunks a warp has requested ahead of the one it reduces) and one mbarrier
+// per stage.  Two CTAs per SM keep 192 KB of logits in flight per SM.
+constexpr int kChunkStages = 3;
+constexpr int kChunkRingBytes = kAccWarps * kChunkStages * kSegTokens * 4;
+constexpr int kChunkSmemBytes = kChunkRingBytes + kAccWarps * kChunkStages * 8;
+
+// kBulk (rows 16-byte aligned, V % 4 == 0): each warp's lane 0 requests its
+// chunks into the warp's ring with 1-D bulk copies, kChunkStages ahead, and
+// the warp reduces them from shared memory; otherwise two register buffers
+// (chunk u + 1 loads while chunk u is reduced).
+template <bool kBulk>
 __global__ void __launch_bounds__(kAccThreads, 2)
 accept_chunks_kernel(const __grid_constant__ AccParams p) {
+  extern __shared__ __align__(128) uint8_t s_ring[];
   // Every input may come from the previous kernel on the stream: wait for
   // it before reading anything, and only then let the finishing kernel be
   // scheduled (so that it too starts after that kernel completed).
   grid_dependency_wait();
   grid_launch_dependents();
-  const int lane = threadIdx.x & 31;
-  const int gw = blockIdx.x * kAccWarps + (threadIdx.x >> 5);
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int gw = blockIdx.x * kAccWarps + warp;
   const int CPR = p.C1;
   const int U = p.B * (p.k + 1) * CPR;  // < 2^31: the host checks V * (k + 1) and B
   const int u0 = static_cast<int>((long long)gw * U / p.NW1);
@@ -885,14 +898,10 @@ accept_chunks_kernel(const __grid_constant__ AccParams p) {
   if (u0 >= u1) return;
   RunState st;
   run_begin(p, st, u0 / CPR, u0 % CPR);
-  // two register buffers: chunk u + 1 is loading while chunk u is reduced
-  float4 xa[8], xb[8];
-  load_chunk(p, st.row, st.c, lane, xa);
-  auto step = [&](int u, const float4 (&cur)[8], float4 (&nxt)[8]) {
+  // the next chunk: the row boundary ends the run
+  auto advance = [&](int u) {
     int nrow = st.row, nc = st.c + 1;
     if (nc == CPR) { nc = 0; ++nrow; }
-    if (u + 1 < u1) load_chunk(p, nrow, nc, lane, nxt);
-    run_chunk(st, lane, cur);
     if (nc == 0 || u + 1 == u1) {
       run_end(p, st, lane, gw, U);
       if (u + 1 < u1) run_begin(p, st, nrow, 0);
@@ -900,9 +909,87 @@ accept_chunks_kernel(const __grid_constant__ AccParams p) {
       st.c = nc;
     }
   };
-  for (int u = u0; u < u1; u += 2) {
-    step(u, xa, xb);
-    if (u + 1 < u1) step(u + 1, xb, xa);
+  if constexpr (kBulk) {
+    const float4 *ring = reinterpret_cast<const float4 *>(s_ring + warp * kChunkStages * kSegTokens * 4);
+    const uint32_t ring_s = smem_addr(ring);
+    const uint32_t bar0 = smem_addr(s_ring + kChunkRingBytes) + static_cast<uint32_t>(warp * kChunkStages * 8);
+    if (lane == 0) {
+#pragma unroll 1
+      for (int s = 0; s < kChunkStages; ++s) mbar_init(bar0 + 8u * s, 1);
+      fence_mbar_init();
+    }
+    __syncwarp();
+    // lane 0: chunk u (row u / CPR, tokens from (u % CPR) * 1024) into stage s
+    auto request = [&](int u, int s) {
+      const int row = u / CPR, c = u - row * CPR;
+      const int n = min(kSegTokens, p.V - c * kSegTokens);
+      const uint32_t bytes = static_cast<uint32_t>(n) * 4u;
+      mbar_arrive_expect_tx(bar0 + 8u * s, bytes);
+      bulk_copy_g2s(ring_s + static_cast<uint32_t>(s * kSegTokens * 4),
+                    p.logits + (size_t)row * p.V + (size_t)c * kSegTokens, bytes, bar0 + 8u * s);
+    };
+    if (lane == 0) {
+#pragma unroll 1
+      for (int s = 0; s < kChunkStages && u0 + s < u1; ++s) request(u0 + s, s);
+    }
+    int issued = min(kChunkStages, u1 - u0);
+#pragma unroll 1
+    for (int u = u0; u < u1; ++u) {
+      const int i = u - u0, s = i % kChunkStages;
+      const bool ok = mbar_wait_bounded(bar0 + 8u * s, static_cast<uint32_t>(i / kChunkStages) & 1u);
+      if (!__all_sync(0xffffffffu, ok)) {
+        // a copy never completed (not expected): flag it, wait (bounded)
+        // for the other requested stages, and stop this warp
+        if (lane == 0) {
+          set_status(p.status, SF_DEVICE_TIMEOUT);
+#pragma unroll 1
+          for (int x = i + 1; x < issued; ++x)
+            (void)mbar_wait_bounded(bar0 + 8u * (x % kChunkStages), static_cast<uint32_t>(x / kChunkStages) & 1u);
+        }
+        return;
+      }
+      float4 x[8];
+#pragma unroll
+      for (int t = 0; t < 8; ++t) x[t] = ring[s * (kSegTokens / 4) + 32 * t + lane];
+      if ((st.c + 1) * kSegTokens > p.V) {
+        // the row's last chunk: tokens at or past V were not copied
+#pragma unroll
+        for (int t = 0; t < 8; ++t) {
+          const int e = st.c * kSegTokens + 128 * t + 4 * lane;
+          if (e >= p.V) x[t].x = -INFINITY;
+          if (e + 1 >= p.V) x[t].y = -INFINITY;
+          if (e + 2 >= p.V) x[t].z = -INFINITY;
+          if (e + 3 >= p.V) x[t].w = -INFINITY;
+        }
+      }
+      run_chunk(st, lane, x);
+      // the stage's reads are complete (their values are consumed): the
+      // next request may overwrite it
+      __syncwarp();
+      if (issued < u1 - u0 && i + kChunkStages == issued) {
+        if (lane == 0) {
+          fence_proxy_async_smem();
+          request(u0 + issued, s);
+        }
+        ++issued;
+      }
+      advance(u);
+    }
+  } else {
+    // two register buffers: chunk u + 1 is loading while chunk u is reduced
+    float4 xa[8], xb[8];
+    load_chunk(p, st.row, st.c, lane, xa);
+    auto step = [&](int u, const float4 (&cur)[8], float4 (&nxt)[8]) {
+      int nrow = st.row, nc = st.c + 1;
+      if (nc == CPR) { nc = 0; ++nrow; }
+      if (u + 1 < u1) load_chunk(p, nrow, nc, lane, nxt);
+      run_chunk(st, lane, cur);
+      advance(u);
+    };
+    for (int u = u0; u < u1; u += 2) {
+      step(u, xa, xb);
+      if (u + 1 < u1) step(u + 1, xb, xa);
+    }
   }
 }
 
@@ -1081,6 +1168,23 @@ static int cluster_setup(int cs, bool *ok) {
   return SF_OK;
 }
 
+// Raises the bulk-copy chunk kernel's dynamic shared memory limit once per
+// device.
+static int chunks_setup(int device) {
+  static std::mutex mu;
+  static bool done[64] = {};
+  if (device < 0 || device >= 64) return fail(SF_ERR_UNSUPPORTED, "device ordinal %d", device);
+  std::lock_guard<std::mutex> lock(mu);
+  if (!done[device]) {
+    const cudaError_t e = cudaFuncSetAttribute(accept_chunks_kernel<true>,
+                                               cudaFuncAttributeMaxDynamicSharedMemorySize, kChunkSmemBytes);
+    if (e != cudaSuccess)
+      return fail(SF_ERR_CUDA, "cudaFuncSetAttribute (accept chunks): %s", cudaGetErrorString(e));
+    done[device] = true;
+  }
+  return SF_OK;
+}
+
 static int check_accept_shapes(int B, int k, int V) {
   if (B < 1 || B > SF_MAX_BATCH) return fail(SF_ERR_INVALID_ARG, "B=%d outside [1, %d]", B, SF_MAX_BATCH);
   if (k < 1 || k > SF_MAX_DRAFT) return fail(SF_ERR_INVALID_ARG, "k=%d outside [1, %d]", k, SF_MAX_DRAFT);
@@ -1201,13 +1305,19 @@ int sf_accept(const float *target_logits, const float *draft_probs,
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(static_cast<unsigned>(ctas));
   cfg.blockDim = dim3(kAccThreads);
-  cfg.dynamicSmemBytes = 0;
+  cfg.dynamicSmemBytes = prm.vec4 ? kChunkSmemBytes : 0;
   cfg.stream = stream;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  cudaError_t e = cudaLaunchKernelEx(&cfg, accept_chunks_kernel, prm);
+  if (prm.vec4) {
+    st = chunks_setup(dev.ordinal);
+    if (st != SF_OK) return st;
+  }
+  cudaError_t e = prm.vec4 ? cudaLaunchKernelEx(&cfg, accept_chunks_kernel<true>, prm)
+                           : cudaLaunchKernelEx(&cfg, accept_chunks_kernel<false>, prm);
   if (e != cudaSuccess) return fail(SF_ERR_CUDA, "accept chunks launch: %s", cudaGetErrorString(e));
   cfg.gridDim = dim3(plan.C2, B);
+  cfg.dynamicSmemBytes = 0;
   e = cudaLaunchKernelEx(&cfg, accept_finish_kernel, prm);
   if (e != cudaSuccess) return fail(SF_ERR_CUDA, "accept finish launch: %s", cudaGetErrorString(e));
   return SF_OK;
