@@ -577,7 +577,7 @@ def time_workload(name, dev, stream, capture, peak, reps=20):
             "kv_gbs": kv_gbs, "frac": kv_gbs / peak,
             "layers_rotated": n_layers, "attention_finite": finite,
             "accept_kernels": (["accept_cluster_kernel"] if sfv.accept_kernel_launches(
-                wl.B, wl.k, wl.V) == 1 else ["accept_chunks_kernel", "accept_finish_kernel"]),
+                wl.B, wl.k, wl.V) == 1 else ["accept_chunks_kernel", "accept_draw_kernel"]),
             "accept_us": acc_us, "accept_algorithmic_bytes": acc_bytes, "accept_gbs": acc_gbs,
             "accept_frac": acc_gbs / peak, "accept_input_copies_rotated": n_copies,
             "mean_accepted": float(n_acc.float().mean().item()),

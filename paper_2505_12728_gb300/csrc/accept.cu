@@ -17,9 +17,10 @@
 //  * V <= 16 x 2048: accept_cluster_kernel, one thread-block cluster per
 //    sequence, the phases separated by cluster barriers (below);
 //  * larger V: accept_chunks_kernel (every row in 1024-token chunks over
-//    all SMs, row records combined by the warp that completes a row) then
-//    accept_finish_kernel (decisions, then the residual draw in C2 chunks of
-//    row j, the last CTA of a sequence scanning for u_k * S);
+//    all SMs; the warp that completes a row combines its run records, the
+//    one that completes a sequence takes the decisions) then
+//    accept_draw_kernel (the residual draw in C2 CTAs per sequence over row
+//    j, the last CTA of a sequence scanning for u_k * S);
 //  * behind the fused LM head, whose projection already left per-CTA row
 //    statistics: accept_decide_kernel then accept_draw_kernel.
 // Every launch uses programmatic stream serialisation: a kernel is resident
@@ -81,6 +82,8 @@ struct AccParams {
   float *ratio;            // [B][k] or null
   uint32_t *status;
   uint32_t *draw_tickets;  // [B]
+  uint32_t *row_tickets;   // [B][k+1]: runs of a row whose record is written (chunk kernel)
+  uint32_t *seq_tickets;   // [B]: rows of a sequence whose statistics are final
   RowStat *runs;           // [B][k+1][C1]: per row, one record per run of the chunk kernel
   RowStat *rows;           // [B][k+1]
   SeqState *seqs;          // [B]
@@ -752,11 +755,11 @@ accept_draw_kernel(const __grid_constant__ AccParams p) {
 // and writes one run record; the runs of row R are stored in warp order, so
 // that run t of the row is the one of warp warp_of(R C1) + t.
 //
-// accept_finish_kernel, grid (C2, B): every CTA of sequence b combines the
-// run records of the k+1 rows (one warp per row, in run order), reads the
-// draft tokens' logits and probabilities, takes the k decisions (the same
-// device function as the other paths; CTA 0 writes the outputs) and, for a
-// sampled sequence, does its part of the residual draw (draw_residual).
+// The warp that writes a row's last run record (a ticket per row) combines
+// the row's runs in run order into its final statistics; the warp that
+// finalises a sequence's k + 1 rows (a ticket per sequence) takes the k
+// decisions.  accept_draw_kernel, grid (C2, B), then draws the token of row
+// j for the sampled sequences.
 // --------------------------------------------------------------------------
 
 // The warp of the chunk kernel owning chunk u: the largest g with
@@ -850,9 +853,86 @@ __device__ __forceinline__ void run_chunk(RunState &st, int lane, const float4 (
   ++st.len;
 }
 
-// Ends the warp's run: combines the lanes and writes the run's record.
-__device__ __forceinline__ void run_end(const AccParams &p, const RunState &st, int lane, int gw,
-                                        int U) {
+__device__ __forceinline__ RowStat combine_runs(const AccParams &p, int row, float tau,
+                                                bool greedy);
+
+// The k accept/reject decisions of sequence b by one warp, from the final
+// row statistics (lane i < k tests draft i, exactly as decide_sequence
+// does); writes every output except, for a sampled sequence, out_tokens[j],
+// which the draw kernel writes.
+__device__ void decide_warp(const AccParams &p, int b) {
+  const int lane = threadIdx.x & 31, k = p.k, V = p.V;
+  const float tau = p.tau[b];
+  const bool greedy = !(tau > 0.0f);
+  const RowStat *rows = p.rows + (size_t)b * (k + 1);
+  float rm = 0.f;
+  int rarg = -1;
+  ff rS = ff_of(0.f);
+  if (lane <= k) {
+    const float4 v = __ldcg(reinterpret_cast<const float4 *>(rows + lane));
+    rm = v.x;
+    rarg = __float_as_int(v.y);
+    rS = ff{v.z, v.w};
+  }
+  int tok = -1;
+  float u = 0.f, lx = 0.f, qx = 0.f;
+  bool in_range = false;
+  if (lane < k) {
+    tok = p.tokens[(size_t)b * k + lane];
+    u = p.u[(size_t)b * (k + 1) + lane];
+    in_range = tok >= 0 && tok < V;
+    if (in_range) {
+      lx = p.logits[((size_t)b * (k + 1) + lane) * V + tok];
+      qx = p.q[((size_t)b * k + lane) * V + tok];
+    }
+  }
+  int acc = 0;
+  if (lane < k) {
+    float ratio = 0.f;
+    if (!in_range) {
+      set_status(p.status, SF_DEVICE_BAD_TOKEN);  // treated as a rejection
+    } else if (greedy) {
+      acc = tok == rarg;
+      ratio = acc ? 1.f : 0.f;
+    } else {
+      // p(x) = exp((l_x - m) / tau) / S; accept iff u * q(x) < p(x), with the
+      // product u * q kept exactly as float-float
+      const float px = ff_div_to_f(exp_diff_accurate(lx, rm, tau), rS);
+      const float uq = __fmul_rn(u, qx);
+      const ff uqf = ff{uq, __fmaf_rn(u, qx, -uq)};
+      acc = ff_lt(uqf, ff_of(px)) ? 1 : 0;
+      ratio = qx > 0.f ? fminf(1.f, __fdiv_rn(px, qx)) : 1.f;
+    }
+    if (p.ratio) p.ratio[(size_t)b * k + lane] = ratio;
+  }
+  const unsigned rejected = __ballot_sync(0xffffffffu, lane < k && !acc);
+  const int j = rejected ? __ffs(rejected) - 1 : k;
+  const int arg_j = __shfl_sync(0xffffffffu, rarg, j);
+  if (lane <= k) {
+    int v = -1;
+    if (lane < j) v = tok;
+    else if (lane == j && greedy) v = arg_j;
+    if (!(lane == j && !greedy)) p.out_tokens[(size_t)b * (k + 1) + lane] = v;
+  }
+  if (lane == 0) {
+    p.num_accepted[b] = j;
+    p.seqs[b].j = j;
+  }
+}
+
+// A run record whose row ticket is taken but not yet looked at (the
+// atomic's result is read one run later, so its latency hides behind the
+// next run's streaming).
+struct PendingTicket {
+  int row;          // -1: none
+  int n_runs;       // runs of the row
+  uint32_t ticket;  // lane 0: the row ticket before this warp's add
+};
+
+// Ends the warp's run: combines the lanes, writes the run's record and
+// takes the row's ticket (lane 0; one atomic per run; nobody waits).
+__device__ __forceinline__ PendingTicket run_end(const AccParams &p, const RunState &st, int lane,
+                                                 int gw, int U) {
   float wm = st.lm;
   int wi = st.li;
   warp_argmax(wm, wi);
@@ -862,11 +942,37 @@ __device__ __forceinline__ void run_end(const AccParams &p, const RunState &st, 
     if (ff_pos(st.lS)) mine = ff_mul(st.lS, exp_diff_accurate(st.lm, wm, st.tau));
     S = warp_sum_ff(mine);
   }
+  const int CPR = p.C1;
+  const int g0 = warp_of(st.row * CPR, U, p.NW1);
+  PendingTicket pt{st.row, warp_of(st.row * CPR + CPR - 1, U, p.NW1) - g0 + 1, 0u};
   if (lane == 0) {
-    const int CPR = p.C1;
-    const int t = gw - warp_of(st.row * CPR, U, p.NW1);  // the run's place in its row
-    p.runs[(size_t)st.row * CPR + t] = RowStat{wm, wi, S};
+    p.runs[(size_t)st.row * CPR + (gw - g0)] = RowStat{wm, wi, S};  // run gw - g0 of its row
+    // the release covers the record; the acquire, the other runs' records
+    pt.ticket = atom_add_acq_rel_gpu(p.row_tickets + pt.row, 1u);
   }
+  return pt;
+}
+
+// Looks at a taken row ticket: the warp that wrote the row's last record
+// combines the row's runs in run order into its final statistics, and the
+// warp that finalises a sequence's k + 1 rows takes its decisions.
+__device__ __forceinline__ void resolve_ticket(const AccParams &p, const PendingTicket &pt, int lane) {
+  const bool last = __shfl_sync(0xffffffffu, pt.ticket == static_cast<uint32_t>(pt.n_runs - 1), 0);
+  if (!last) return;
+  __syncwarp();
+  const float tau = __ldg(p.tau + pt.row / (p.k + 1));
+  const RowStat rs = combine_runs(p, pt.row, tau, !(tau > 0.0f));
+  const int b = pt.row / (p.k + 1);
+  uint32_t last_row = 0;
+  if (lane == 0) {
+    p.rows[pt.row] = rs;
+    p.row_tickets[pt.row] = 0u;  // zero again for the next call
+    last_row = atom_add_acq_rel_gpu(p.seq_tickets + b, 1u) == static_cast<uint32_t>(p.k);
+  }
+  if (!__shfl_sync(0xffffffffu, last_row, 0)) return;
+  __syncwarp();
+  decide_warp(p, b);
+  if (lane == 0) p.seq_tickets[b] = 0u;
 }
 
 // Chunk ring of the bulk-copy path: kChunkStages 4 KB stages per warp (the
@@ -898,12 +1004,15 @@ accept_chunks_kernel(const __grid_constant__ AccParams p) {
   if (u0 >= u1) return;
   RunState st;
   run_begin(p, st, u0 / CPR, u0 % CPR);
-  // the next chunk: the row boundary ends the run
+  PendingTicket pend{-1, 0, 0u};
+  // the next chunk: the row boundary ends the run (and looks at the
+  // previous run's ticket)
   auto advance = [&](int u) {
     int nrow = st.row, nc = st.c + 1;
     if (nc == CPR) { nc = 0; ++nrow; }
     if (nc == 0 || u + 1 == u1) {
-      run_end(p, st, lane, gw, U);
+      const PendingTicket now = run_end(p, st, lane, gw, U);
+      resolve_ticket(p, now, lane);
       if (u + 1 < u1) run_begin(p, st, nrow, 0);
     } else {
       st.c = nc;
@@ -1043,47 +1152,6 @@ __device__ __forceinline__ RowStat combine_runs(const AccParams &p, int row, flo
   return RowStat{mv, mi, Sr};
 }
 
-__global__ void __launch_bounds__(kAccThreads, 3)
-accept_finish_kernel(const __grid_constant__ AccParams p) {
-  __shared__ int s_acc[SF_MAX_DRAFT], s_j;
-  __shared__ float s_rm[SF_MAX_DRAFT + 1], s_rlx[SF_MAX_DRAFT + 1], s_rqx[SF_MAX_DRAFT + 1];
-  __shared__ int s_rarg[SF_MAX_DRAFT + 1], s_rhx[SF_MAX_DRAFT + 1];
-  __shared__ ff s_rS[SF_MAX_DRAFT + 1];
-  const int c = blockIdx.x, b = blockIdx.y, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  const int k = p.k, V = p.V;
-  grid_dependency_wait();  // the run records (and every input) follow the previous kernel
-  grid_launch_dependents();
-  const float tau = p.tau[b];
-  const bool greedy = !(tau > 0.0f);
-  int my_tok = -1;
-  float my_u = 0.f;
-  if (tid < k) {
-    // draft token i's logit and draft probability, read directly
-    my_tok = p.tokens[(size_t)b * k + tid];
-    my_u = p.u[(size_t)b * (k + 1) + tid];
-    const bool ok = my_tok >= 0 && my_tok < V;
-    s_rlx[tid] = ok ? p.logits[((size_t)b * (k + 1) + tid) * V + my_tok] : 0.f;
-    s_rqx[tid] = ok ? p.q[((size_t)b * k + tid) * V + my_tok] : 0.f;
-    s_rhx[tid] = ok ? 1 : 0;
-  }
-  for (int r = warp; r <= k; r += kAccWarps) {
-    const RowStat rs = combine_runs(p, b * (k + 1) + r, tau, greedy);
-    if (lane == 0) {
-      s_rm[r] = rs.m;
-      s_rarg[r] = rs.arg;
-      s_rS[r] = rs.S;
-    }
-  }
-  __syncthreads();
-  decide_sequence(p, b, greedy, tau, my_tok, my_u, s_rm, s_rarg, s_rS, s_rlx, s_rqx, s_rhx, s_acc,
-                  c == 0, &s_j);
-  __syncthreads();
-  if (greedy) return;  // CTA 0 wrote the argmax of row j
-  const int j = s_j;
-  const float u_k = p.u[(size_t)b * (k + 1) + k];
-  draw_residual(p, b, c, j, RowStat{s_rm[j], s_rarg[j], s_rS[j]}, tau, u_k);
-}
-
 // --------------------------------------------------------------------------
 // host side
 // --------------------------------------------------------------------------
@@ -1092,7 +1160,7 @@ struct AccPlan {
 };
 
 struct AccLayout {
-  size_t draw_tickets, runs, rows, seqs, parts, total;
+  size_t draw_tickets, row_tickets, seq_tickets, runs, rows, seqs, parts, total;
 };
 
 static int plan_accept(int V, AccPlan *plan) {
@@ -1106,6 +1174,8 @@ static AccLayout acc_layout(int B, int k, const AccPlan &pl) {
   const size_t R = (size_t)B * (k + 1);
   size_t off = 256;
   l.draw_tickets = off; off = round_up(off + 4 * (size_t)B, 256);
+  l.row_tickets = off; off = round_up(off + 4 * R, 256);
+  l.seq_tickets = off; off = round_up(off + 4 * (size_t)B, 256);
   l.runs = off; off = round_up(off + sizeof(RowStat) * R * pl.C1, 256);
   l.rows = off; off = round_up(off + sizeof(RowStat) * R, 256);
   l.seqs = off; off = round_up(off + sizeof(SeqState) * (size_t)B, 256);
@@ -1250,6 +1320,8 @@ int sf_accept(const float *target_logits, const float *draft_probs,
   prm.ratio = accept_ratio;
   prm.status = reinterpret_cast<uint32_t *>(ws);
   prm.draw_tickets = reinterpret_cast<uint32_t *>(ws + lay.draw_tickets);
+  prm.row_tickets = reinterpret_cast<uint32_t *>(ws + lay.row_tickets);
+  prm.seq_tickets = reinterpret_cast<uint32_t *>(ws + lay.seq_tickets);
   prm.runs = reinterpret_cast<RowStat *>(ws + lay.runs);
   prm.rows = reinterpret_cast<RowStat *>(ws + lay.rows);
   prm.seqs = reinterpret_cast<SeqState *>(ws + lay.seqs);
@@ -1298,10 +1370,13 @@ int sf_accept(const float *target_logits, const float *draft_probs,
   DeviceInfo dev;
   st = current_device(&dev);
   if (st != SF_OK) return st;
+  // at most one warp per chunk, so that every warp owns at least one chunk
+  // (a row's runs are then exactly the warps between its first and last
+  // chunk's owners), and at most two CTAs per SM
   const long long units = (long long)B * (k + 1) * plan.C1;
-  long long ctas = (units + kAccWarps - 1) / kAccWarps;
-  if (ctas > 2LL * dev.sm_count) ctas = 2LL * dev.sm_count;  // two CTAs per SM
-  prm.NW1 = static_cast<int>(ctas) * kAccWarps;
+  long long nw = units < 2LL * dev.sm_count * kAccWarps ? units : 2LL * dev.sm_count * kAccWarps;
+  const long long ctas = (nw + kAccWarps - 1) / kAccWarps;
+  prm.NW1 = static_cast<int>(nw);
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(static_cast<unsigned>(ctas));
   cfg.blockDim = dim3(kAccThreads);
@@ -1318,8 +1393,8 @@ int sf_accept(const float *target_logits, const float *draft_probs,
   if (e != cudaSuccess) return fail(SF_ERR_CUDA, "accept chunks launch: %s", cudaGetErrorString(e));
   cfg.gridDim = dim3(plan.C2, B);
   cfg.dynamicSmemBytes = 0;
-  e = cudaLaunchKernelEx(&cfg, accept_finish_kernel, prm);
-  if (e != cudaSuccess) return fail(SF_ERR_CUDA, "accept finish launch: %s", cudaGetErrorString(e));
+  e = cudaLaunchKernelEx(&cfg, accept_draw_kernel, prm);
+  if (e != cudaSuccess) return fail(SF_ERR_CUDA, "accept draw launch: %s", cudaGetErrorString(e));
   return SF_OK;
 }
 
@@ -1384,6 +1459,8 @@ int sf_verify_lm_head_accept(const void *hidden, const void *weight, const float
   prm.out_tokens = out_tokens;
   prm.ratio = accept_ratio;
   prm.status = reinterpret_cast<uint32_t *>(ws);
+  prm.row_tickets = reinterpret_cast<uint32_t *>(ws + lay.row_tickets);
+  prm.seq_tickets = reinterpret_cast<uint32_t *>(ws + lay.seq_tickets);
   prm.draw_tickets = reinterpret_cast<uint32_t *>(ws + lay.draw_tickets);
   prm.runs = reinterpret_cast<RowStat *>(ws + lay.runs);
   prm.rows = reinterpret_cast<RowStat *>(ws + lay.rows);

@@ -183,6 +183,23 @@ def test_warp_runs_longer_than_32_chunks(oracle_mod):
     _check(oracle_mod, inp, max_excluded_frac=0.1)
 
 
+@pytest.mark.parametrize("B,k,V", [(1, 1, 32769), (1, 2, 40000), (3, 1, 33000), (2, 3, 65537)])
+def test_fewer_chunks_than_warps_all_negative_logits(oracle_mod, B, k, V):
+    # Few 1024-token chunks in all (B (k+1) ceil(V/1024) of 66 to 520): the
+    # chunk kernel then runs one warp per chunk, and every row's run records
+    # come from the warps that own its chunks.  Logits far below zero make
+    # any stale or zero record visible: it would win the row maximum.
+    ws = sfv.new_workspace(sfv.accept_workspace_size(B, k, V))
+    for mode in ("greedy", "sampling"):
+        inp = make_accept_case(B, k, V, seed=V + k, mode=mode)
+        inp.target_logits -= np.float32(50.0)
+        ref = oracle_accept(oracle_mod, inp)
+        # twice on one workspace: the row and sequence tickets return to zero
+        for _ in range(2):
+            n, toks, ratio = run_accept(inp, workspace=ws)
+            assert compare_accept(ref, n, toks, ratio) <= 1
+
+
 def test_out_of_range_draft_token_is_flagged_and_rejected(oracle_mod):
     inp = make_accept_case(4, 3, 1000, seed=8)
     inp.draft_tokens[2, 1] = 5000
@@ -206,7 +223,7 @@ def test_repeated_calls_are_bit_identical():
 
 def test_kernel_launch_counts_follow_the_vocabulary():
     # one cluster kernel while a row fits 16 slices of 2048 tokens, else the
-    # chunk and finish kernels
+    # chunk kernel (statistics and decisions) and draw kernel
     assert sfv.accept_kernel_launches(1, 5, 32000) == 1
     assert sfv.accept_kernel_launches(4, 8, 32768) == 1
     assert sfv.accept_kernel_launches(4, 8, 32769) == 2
