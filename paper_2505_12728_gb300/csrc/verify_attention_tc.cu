@@ -612,9 +612,20 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
         }
         // this lane's keys kap*KPL .. kap*KPL + KPL-1 (raw scores; the
         // scale, > 0, is applied to the maximum and folded into the exponent)
-        float mx = -INFINITY;
+        // tile maximum as a tree (a chain of KPL dependent max operations
+        // is ~5 cycles each on the softmax's critical path)
+        float mx;
+        {
+          float t[KPL / 2];
 #pragma unroll
-        for (int c = 0; c < KPL; ++c) mx = fmaxf(mx, __uint_as_float(sv[c]));
+          for (int c = 0; c < KPL / 2; ++c) t[c] = fmaxf(__uint_as_float(sv[2 * c]), __uint_as_float(sv[2 * c + 1]));
+#pragma unroll
+          for (int w = KPL / 4; w >= 1; w >>= 1) {
+#pragma unroll
+            for (int c = 0; c < w; ++c) t[c] = fmaxf(t[c], t[c + w]);
+          }
+          mx = t[0];
+        }
         const int key0 = tile_pos + kap * KPL;
         if (key0 + KPL - 1 > lim) {
           // causal mask of the draft block, positions past the end, padding rows
@@ -633,16 +644,22 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
           ref = mx;
         }
         const float mu = ref == -INFINITY ? 0.f : ref;
-        float rs = 0.f;
         uint32_t mine[KPL / 2], mine_lo[KPL / 2];
+        float ps[KPL / 2];  // pair sums, added as a tree below
 #pragma unroll
         for (int c2 = 0; c2 < KPL / 2; ++c2) {
           const float p0 = fast_exp2(fmaf(__uint_as_float(sv[2 * c2]), p.scale_log2, -mu));
           const float p1 = fast_exp2(fmaf(__uint_as_float(sv[2 * c2 + 1]), p.scale_log2, -mu));
-          rs += p0 + p1;
+          ps[c2] = p0 + p1;
           if (split_p) split_bf16x2(p0, p1, mine[c2], mine_lo[c2]);
           else mine[c2] = pack_bf16x2(p0, p1);
         }
+#pragma unroll
+        for (int w = KPL / 4; w >= 1; w >>= 1) {
+#pragma unroll
+          for (int c = 0; c < w; ++c) ps[c] += ps[c + w];
+        }
+        const float rs = ps[0];
         l_run = l_run * alpha + rs;
         if (__any_sync(0xffffffffu, alpha != 1.f)) {
           // O *= alpha after the P V of tile n-1 (it > 0 here: the first
