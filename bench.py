@@ -171,6 +171,53 @@ def attention_kernel(wl):
         else "verify_attention_kernel"
 
 
+def tc_merge_partial_bytes(wl, seq_lens, sm_count):
+    """Bytes of the tcgen05 kernel's split partials (fp32 O, max and sum per
+    row of each piece of a split segment, written once and read once by the
+    merge kernel), from the partition rule the kernel applies on the device
+    with one CTA per SM: the segment-aligned partition when its piece length
+    is within 3 tiles of the balanced share, else the balanced one.  None for
+    shapes of the mma.sync kernel (at most 16 rows per KV head), which merges
+    through distributed shared memory or a last-CTA merge."""
+    R = wl.rows * (wl.H_q // wl.H_kv)
+    if R <= 16:
+        return None
+    tiles = [(int(t) + 63) // 64 for t in seq_lens]
+    Tot = wl.H_kv * sum(tiles)
+    G = min(Tot, sm_count)
+    S = wl.B * wl.H_kv
+    pieces = None
+    if sm_count > S:
+        Ta = -(-Tot // (sm_count - S))
+        Tmin = -(-Tot // sm_count)
+        if Ta <= Tmin + 3:
+            for cand in range(Tmin, Ta):
+                if wl.H_kv * sum(-(-t // cand) for t in tiles) <= sm_count:
+                    Ta = cand
+                    break
+            pieces = [-(-t // Ta) for t in tiles for _ in range(wl.H_kv)]
+    if pieces is None:
+        q, r = divmod(Tot, G)
+        start = lambda c: c * q + (c * r) // G
+        def owner(t):
+            lo, hi = 0, G - 1
+            while lo < hi:
+                mid = (lo + hi + 1) // 2
+                if start(mid) <= t:
+                    lo = mid
+                else:
+                    hi = mid - 1
+            return lo
+        pieces, base = [], 0
+        for t in tiles:
+            for h in range(wl.H_kv):
+                first = base + h * t
+                pieces.append(owner(first + t - 1) - owner(first) + 1)
+            base += wl.H_kv * t
+    per_piece = (R * wl.d + 2 * R) * 4
+    return 2 * per_piece * sum(n for n in pieces if n > 1)
+
+
 def profiled_traffic(kernel_sources, profile):
     """DRAM bytes per launch from a committed ncu summary, or None when the
     kernel's sources changed since the counters were taken."""
@@ -243,12 +290,39 @@ def cpu_baseline(wl, att, acc, budget_s=12.0):
         if time.perf_counter() - start > budget_s or layers_done >= att.layers:
             break
     step_s = wl.layers * (t_att / layers_done) + t_acc / n_acc
+    # the same oracle on one thread: one attention layer and one acceptance
+    oracle.set_threads(1)
+    try:
+        a1, c1 = time_oracle_step_sample(wl, att, acc, 0)
+    finally:
+        oracle.set_threads(0)
+    step1_s = wl.layers * a1 + c1
     return {"value": wl.B * wl.k / step_s, "unit": UNIT, "cores": oracle_cores(),
             "kind": "oracle",
             "sample": f"fp64 C oracle on the host: {layers_done} of {wl.layers} attention layers "
                       f"and {n_acc} acceptance passes of the {wl.name} workload, scaled to one "
                       f"full step ({step_s * 1e3:.1f} ms)",
-            "step_ms": step_s * 1e3}
+            "step_ms": step_s * 1e3,
+            "value_1thread": wl.B * wl.k / step1_s, "step_ms_1thread": step1_s * 1e3,
+            "cpu_model": cpu_model()}
+
+
+def cpu_model() -> str:
+    """The host CPU's name as /proc/cpuinfo gives it (model name on x86,
+    implementer and part on Arm), with the machine type."""
+    import platform
+    fields = {}
+    try:
+        with open("/proc/cpuinfo") as f:
+            for line in f:
+                if ":" in line:
+                    k, v = line.split(":", 1)
+                    fields.setdefault(k.strip(), v.strip())
+    except OSError:
+        pass
+    name = fields.get("model name") or " ".join(
+        f"{k} {fields[k]}" for k in ("CPU implementer", "CPU part") if k in fields)
+    return f"{name or platform.processor() or 'unknown'} ({platform.machine()}, {os.cpu_count()} cores)"
 
 
 def run_reference(args):
@@ -567,6 +641,12 @@ def time_workload(name, dev, stream, capture, peak, reps=20):
     acc_us = timed(acc_all, n_copies)
     sampling_rows = int(np.sum(acc.temperature > 0))
     acc_bytes = accept_bytes(wl, sampling_rows)
+    # the data-dependent minimum: the logits rows 0..min(j, k) of each
+    # sequence, and row j of q where a sampled sequence rejected draft j
+    j = n_acc.cpu().numpy().astype(np.int64)
+    sampled = acc.temperature > 0
+    acc_min_bytes = int((np.minimum(j, wl.k) + 1).sum() * wl.V * 4
+                        + np.sum(sampled & (j < wl.k)) * wl.V * 4)
     kv_gbs = bytes_layer / (att_us * 1e-6) / 1e9
     acc_gbs = acc_bytes / (acc_us * 1e-6) / 1e9
     return {"description": wl.description, "context_tokens": [int(x) for x in seq_np],
@@ -579,6 +659,9 @@ def time_workload(name, dev, stream, capture, peak, reps=20):
             "accept_kernels": (["accept_cluster_kernel"] if sfv.accept_kernel_launches(
                 wl.B, wl.k, wl.V) == 1 else ["accept_chunks_kernel", "accept_draw_kernel"]),
             "accept_us": acc_us, "accept_algorithmic_bytes": acc_bytes, "accept_gbs": acc_gbs,
+            "accept_min_bytes": acc_min_bytes, "accept_min_gbs": acc_min_bytes / (acc_us * 1e-6) / 1e9,
+            "merge_partial_bytes": tc_merge_partial_bytes(
+                wl, seq_np, torch.cuda.get_device_properties(dev).multi_processor_count),
             "accept_frac": acc_gbs / peak, "accept_input_copies_rotated": n_copies,
             "mean_accepted": float(n_acc.float().mean().item()),
             "device_status": att_status | sfv.read_device_status(ws_a)}
@@ -726,6 +809,19 @@ def run_ours(args):
     torch.cuda.synchronize()
     att_ms = [ev[s][0].elapsed_time(ev[s][1]) for s in range(args.steps)]
     acc_ms = [ev[s][1].elapsed_time(ev[s][2]) for s in range(args.steps)]
+
+    # ---- per-step distribution: a second pass of the step, an event after
+    # every step (the timed region above has none between steps) ----
+    evs = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps + 1)]
+    evs[0].record(stream)
+    for s in range(args.steps):
+        run_step()
+        evs[s + 1].record(stream)
+    torch.cuda.synchronize()
+    per_step = sorted(evs[s].elapsed_time(evs[s + 1]) * 1e3 for s in range(args.steps))
+    pick = lambda fr: per_step[min(len(per_step) - 1, int(round(fr * (len(per_step) - 1))))]
+    step_dist = {"p10": pick(0.1), "median": pick(0.5), "p90": pick(0.9), "unit": "us",
+                 "steps": args.steps}
     ms_per_step = total_ms / args.steps
     tokens = wl.B * wl.k * world * args.steps
     value = tokens / (total_ms / 1e3)
@@ -845,6 +941,7 @@ def run_ours(args):
         "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
         "config": workload_config(wl, att.seq_lens),
         "verify_step_us": ms_per_step * 1e3,
+        "verify_step_us_distribution": step_dist,
         "attention_us_per_layer": att_launch_ms * 1e3,
         "accept_us": others[wl.name]["accept_us"],
         "accept_us_in_step": acc_launch_ms * 1e3,
@@ -880,7 +977,8 @@ def run_ours(args):
         "device_status": status,
     }
     if cpu is not None:
-        line["cpu_baseline"] = {k: cpu[k] for k in ("value", "unit", "cores", "kind", "sample")}
+        line["cpu_baseline"] = {k: cpu[k] for k in ("value", "unit", "cores", "kind", "sample",
+                                                    "value_1thread", "cpu_model")}
     if rank == 0:
         print(json.dumps(line), flush=True)
     if world > 1:

@@ -78,8 +78,16 @@ def _load():
         lib.oracle_sample.restype = I
         lib.oracle_visual_compress.argtypes = [P, P, I, I, I, I, P]
         lib.oracle_visual_compress.restype = I
+        lib.oracle_set_threads.argtypes = [I]
+        lib.oracle_set_threads.restype = None
         _lib = lib
         return lib
+
+
+def set_threads(n: int) -> None:
+    """Threads of the oracle's OpenMP loops (n <= 0: all host cores).  The
+    results do not depend on it."""
+    _load().oracle_set_threads(int(n))
 
 
 def _ptr(a: np.ndarray):

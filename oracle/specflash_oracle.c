@@ -56,6 +56,7 @@
  * acceptance rule; none is "parity unpinned".
  */
 #include <math.h>
+#include <omp.h>
 #include <stdint.h>
 #include <stdlib.h>
 #include <string.h>
@@ -621,4 +622,13 @@ int oracle_visual_compress(const uint16_t *queries, const uint16_t *features, in
     }
     free(s);
     return ORACLE_OK;
+}
+
+/* Threads of the OpenMP loops (the per-row attention loop): n >= 1 sets the
+ * count, n <= 0 restores the default.  Every result is independent of it
+ * (each row is computed by one thread in a fixed order); bench.py times the
+ * oracle on one thread and on all host cores. */
+void oracle_set_threads(int n)
+{
+    omp_set_num_threads(n >= 1 ? n : omp_get_num_procs());
 }
