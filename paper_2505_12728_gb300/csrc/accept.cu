@@ -920,9 +920,8 @@ __device__ void decide_warp(const AccParams &p, int b) {
   }
 }
 
-// A run record whose row ticket is taken but not yet looked at (the
-// atomic's result is read one run later, so its latency hides behind the
-// next run's streaming).
+// A run record whose row ticket is taken: the row, its number of runs and
+// (lane 0) the ticket's value before this warp's add.
 struct PendingTicket {
   int row;          // -1: none
   int n_runs;       // runs of the row
@@ -1004,9 +1003,7 @@ accept_chunks_kernel(const __grid_constant__ AccParams p) {
   if (u0 >= u1) return;
   RunState st;
   run_begin(p, st, u0 / CPR, u0 % CPR);
-  PendingTicket pend{-1, 0, 0u};
-  // the next chunk: the row boundary ends the run (and looks at the
-  // previous run's ticket)
+  // the next chunk: the row boundary ends the run and looks at its ticket
   auto advance = [&](int u) {
     int nrow = st.row, nc = st.c + 1;
     if (nc == CPR) { nc = 0; ++nrow; }
