@@ -628,45 +628,75 @@ __device__ void draw_residual(const AccParams &p, int b, int c, int j, RowStat r
     const float4 v = __ldcg(reinterpret_cast<const float4 *>(parts + cc));
     return pmass ? ff{v.z, v.w} : ff{v.x, v.y};
   };
-  ff total;
-  {
-    ff pr = ff_of(0.f);
-    for (int cc = tid; cc < NS; cc += kAccThreads) pr = ff_add(pr, part_sum(cc, false));
-    total = block_sum(pr, s_d);
-  }
-  const bool use_p = !ff_pos(total);  // residual with no mass (rounding only)
-  if (use_p) {
-    ff pp = ff_of(0.f);
-    for (int cc = tid; cc < NS; cc += kAccThreads) pp = ff_add(pp, part_sum(cc, true));
-    total = block_sum(pp, s_d);
-  }
-  const ff target = ff_mul(total, u_k);
-
-  // segment holding the target: inclusive float-float scan over the segment
-  // sums in order; segment cc covers [excl, incl), and excl of cc is
-  // bit-identical to incl of cc - 1, so the intervals tile [0, total)
+  ff target;
+  bool use_p;
+  int my_last_r = -1, my_last_p = -1;  // one segment per thread: its last indices
   if (tid == 0) { s_seg = INT_MAX; s_base = ff_of(0.f); }
-  ff carry = ff_of(0.f);
-  for (int base = 0; base < NS; base += kAccThreads) {
-    const int cc = base + tid;
-    const ff v = cc < NS ? part_sum(cc, use_p) : ff_of(0.f);
-    ff excl_local, blk_total;
-    const ff incl_local = block_inclusive_scan(v, s_scan, &excl_local, &blk_total);
-    const ff excl = ff_add(carry, excl_local), incl = ff_add(carry, incl_local);
-    if (cc < NS && ff_pos(v) && ff_lt(target, incl) && !ff_lt(target, excl)) atomicMin(&s_seg, cc);
+  if (NS <= kAccThreads) {
+    // one segment per thread: every part is loaded once, and one scan gives
+    // both the segment intervals and the total (its last inclusive value, so
+    // that the intervals tile [0, total) exactly)
+    float4 v0 = make_float4(0.f, 0.f, 0.f, 0.f);
+    if (tid < NS) {
+      v0 = __ldcg(reinterpret_cast<const float4 *>(parts + tid));
+      my_last_r = __ldcg(&parts[tid].last_r);
+      my_last_p = __ldcg(&parts[tid].last_p);
+    }
+    ff v = ff{v0.x, v0.y};
+    ff excl, total;
+    ff incl = block_inclusive_scan(v, s_scan, &excl, &total);
+    use_p = !ff_pos(total);  // residual with no mass (rounding only)
+    if (use_p) {
+      v = ff{v0.z, v0.w};
+      incl = block_inclusive_scan(v, s_scan, &excl, &total);
+    }
+    target = ff_mul(total, u_k);
+    if (tid < NS && ff_pos(v) && ff_lt(target, incl) && !ff_lt(target, excl)) atomicMin(&s_seg, tid);
     __syncthreads();
-    if (s_seg == cc) s_base = excl;
-    carry = ff_add(carry, blk_total);
-    __syncthreads();
-    if (s_seg != INT_MAX) break;
+    if (s_seg == tid) s_base = excl;
+  } else {
+    ff total;
+    {
+      ff pr = ff_of(0.f);
+      for (int cc = tid; cc < NS; cc += kAccThreads) pr = ff_add(pr, part_sum(cc, false));
+      total = block_sum(pr, s_d);
+    }
+    use_p = !ff_pos(total);  // residual with no mass (rounding only)
+    if (use_p) {
+      ff pp = ff_of(0.f);
+      for (int cc = tid; cc < NS; cc += kAccThreads) pp = ff_add(pp, part_sum(cc, true));
+      total = block_sum(pp, s_d);
+    }
+    target = ff_mul(total, u_k);
+    // segment holding the target: inclusive float-float scan over the
+    // segment sums in order; segment cc covers [excl, incl), and excl of cc
+    // is bit-identical to incl of cc - 1, so the intervals tile [0, total)
+    ff carry = ff_of(0.f);
+    for (int base = 0; base < NS; base += kAccThreads) {
+      const int cc = base + tid;
+      const ff v = cc < NS ? part_sum(cc, use_p) : ff_of(0.f);
+      ff excl_local, blk_total;
+      const ff incl_local = block_inclusive_scan(v, s_scan, &excl_local, &blk_total);
+      const ff excl = ff_add(carry, excl_local), incl = ff_add(carry, incl_local);
+      if (cc < NS && ff_pos(v) && ff_lt(target, incl) && !ff_lt(target, excl)) atomicMin(&s_seg, cc);
+      __syncthreads();
+      if (s_seg == cc) s_base = excl;
+      carry = ff_add(carry, blk_total);
+      __syncthreads();
+      if (s_seg != INT_MAX) break;
+    }
   }
   __syncthreads();
   int token = -1;
   if (s_seg == INT_MAX) {
     // u*S at or past the total (rounding): the last token with positive mass
     int last = -1;
-    for (int cc = tid; cc < NS; cc += kAccThreads)
-      last = max(last, use_p ? __ldcg(&parts[cc].last_p) : __ldcg(&parts[cc].last_r));
+    if (NS <= kAccThreads) {
+      last = use_p ? my_last_p : my_last_r;
+    } else {
+      for (int cc = tid; cc < NS; cc += kAccThreads)
+        last = max(last, use_p ? __ldcg(&parts[cc].last_p) : __ldcg(&parts[cc].last_r));
+    }
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) last = max(last, __shfl_xor_sync(0xffffffffu, last, o));
     if (tid == 0) s_token = -1;
