@@ -71,6 +71,31 @@ def test_vocabulary_beyond_the_single_kernel_path(oracle_mod, mode):
     _check(oracle_mod, make_accept_case(3, 4, 200003, seed=17, mode=mode))
 
 
+@pytest.mark.parametrize("V", [300000, 300001])
+@pytest.mark.parametrize("mode", ["sampling", "alternate"])
+def test_vocabulary_beyond_256_segments(oracle_mod, V, mode):
+    # more than 256 segments of 1024 tokens per row: the draw's last CTA
+    # searches the segment sums block by block (one segment per thread
+    # otherwise); V % 4 == 0 streams the logits by bulk copies, V % 4 != 0
+    # through registers
+    _check(oracle_mod, make_accept_case(2, 3, V, seed=V % 97, mode=mode))
+
+
+def test_logits_not_16_byte_aligned(oracle_mod):
+    # logits that start 4 bytes past a 16-byte boundary (V % 4 == 0): the
+    # chunk kernel reads them through registers instead of bulk copies
+    inp = make_accept_case(3, 4, 152064, seed=23, mode="alternate")
+    dev = accept_to_device(inp)
+    n_el = inp.target_logits.size
+    big = torch.empty(n_el + 4, dtype=torch.float32, device="cuda")
+    big[1:1 + n_el].copy_(torch.from_numpy(inp.target_logits.reshape(-1)).cuda())
+    dev["target_logits"] = big[1:1 + n_el].view(inp.target_logits.shape)
+    assert dev["target_logits"].data_ptr() % 16 == 4
+    n, toks, ratio = run_accept(inp, dev=dev)
+    ref = oracle_accept(oracle_mod, inp)
+    assert compare_accept(ref, n, toks, ratio) <= 1
+
+
 @pytest.mark.parametrize("V,k", [(2, 3), (3, 2), (5, 2), (5, 3)])
 def test_brute_force_tiny_vocabularies(oracle_mod, V, k):
     # Every draft tuple in [0, V)^k, each with 64 uniform vectors drawn from
