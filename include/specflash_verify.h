@@ -218,9 +218,8 @@ size_t sf_accept_workspace_size(int B, int k, int V);
 /* Kernels one sf_accept call with these shapes launches on the current      */
 /* device: 1 (a row fits one 16-CTA thread-block cluster, V <= 32768, and    */
 /* such a cluster can be resident) or 2 (statistics and decisions, then the  */
-/* draw); 0 for                                                              */
-/* shapes sf_accept rejects or without a usable CUDA device (sf_last_error  */
-/* says which).  For graph and launch planning.                             */
+/* draw); 0 for shapes sf_accept rejects or without a usable CUDA device     */
+/* (sf_last_error says which).  For graph and launch planning.              */
 int sf_accept_kernel_launches(int B, int k, int V);
 
 int sf_accept(const float *target_logits, const float *draft_probs,
