@@ -173,8 +173,8 @@ def attention_kernel(wl):
 
 def tc_merge_partial_bytes(wl, seq_lens, sm_count):
     """Bytes of the tcgen05 kernel's split partials (fp32 O, max and sum per
-    row of each piece of a split segment, written once and read once by the
-    merge kernel), from the partition rule the kernel applies on the device
+    row of each key-split copy of each piece of a split segment, written once
+    and read once by the merge kernel), from the partition rule the kernel applies on the device
     with one CTA per SM: the segment-aligned partition when its piece length
     is within 3 tiles of the balanced share, else the balanced one.  None for
     shapes of the mma.sync kernel (at most 16 rows per KV head), which merges
@@ -214,7 +214,9 @@ def tc_merge_partial_bytes(wl, seq_lens, sm_count):
                 first = base + h * t
                 pieces.append(owner(first + t - 1) - owner(first) + 1)
             base += wl.H_kv * t
-    per_piece = (R * wl.d + 2 * R) * 4
+    # a split piece writes one partial per key-split copy of its rows
+    copies = 4 if R <= 32 else (2 if R <= 64 else 1)
+    per_piece = copies * (R * wl.d + 2 * R) * 4
     return 2 * per_piece * sum(n for n in pieces if n > 1)
 
 

@@ -815,7 +815,9 @@ static AttnLayout attn_layout(int B, int H_kv, int R, int D, long long G) {
   const size_t segs = (size_t)B * H_kv;
   l.tickets_off = 256;
   l.partials_off = round_up(l.tickets_off + 8 * segs, 256);
-  l.total = round_up(l.partials_off + (size_t)(G + (long long)segs) * partial_slot_floats(R, D) * 4,
+  // the tcgen05 kernel (R > 16) writes one partial per key-split copy
+  const long long copies = R > 16 ? (R <= 32 ? 4 : (R <= 64 ? 2 : 1)) : 1;
+  l.total = round_up(l.partials_off + (size_t)((G + (long long)segs) * copies) * partial_slot_floats(R, D) * 4,
                      256);
   return l;
 }

@@ -23,8 +23,10 @@
 //    softmax, owns keys [kap * KPL, (kap + 1) * KPL) of every 64-key tile
 //    (KPL = 64 / F).  A copy is a whole number of 32-lane quarters, so each
 //    softmax warp reads exactly its keys' score columns.  The repeated rows
-//    cost the 128-row MMAs nothing; the F partial states of a row merge
-//    through shared memory at the end of a piece.
+//    cost the 128-row MMAs nothing.  The F partial states of a row merge
+//    through shared memory when the piece is a whole segment; a split
+//    segment's pieces write one partial per copy and the merge kernel
+//    combines all of them (no exchange on the split kernel's tail).
 //  * Q lives in tensor memory (the A operand of S = Q K^T): each softmax
 //    thread writes its lane's row.  Four S buffers: P = exp2(S') is written
 //    as bf16 over the scores it came from, so Q K^T of tile n+4 (which
@@ -53,8 +55,9 @@
 //    divided by (rows with a handful of visible keys would otherwise show
 //    P's bf16 rounding).
 //  * A piece that covers a whole segment writes bf16 out and the LSE; a
-//    split segment's pieces write fp32 partials to the workspace (O as
-//    [D/4][R] float4, so that a warp's stores are contiguous), which
+//    split segment's pieces write fp32 partials to the workspace, one per
+//    key-split copy (O as [D/4][R] float4, so that a warp's stores are
+//    contiguous), which
 //    verify_tc_merge_kernel combines across the whole GPU right after this
 //    kernel (one CTA merging a segment's ~250 KB of partials alone took
 //    longer than the whole split phase).
@@ -719,6 +722,31 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
         break;
       }
       tc_fence_after_sync();
+      if (pc.n_pieces > 1) {
+        // a split segment: each key-split copy writes its own partial
+        // (relative to its own reference); the merge kernel combines the
+        // n_pieces x F partials, so no exchange between the copies here
+        float *partk = p.partials + ((size_t)(blockIdx.x + pc.seg) * F + kap) * p.slot_stride;
+#pragma unroll 1
+        for (int ch = 0; ch < D / 32; ++ch) {
+          uint32_t ov[32];
+          tmem_ld_32x32b_x32(tl + kTmemO + ch * 32, ov);  // warp-wide: every lane loads
+          if (valid) {
+            float4 *dst = reinterpret_cast<float4 *>(partk) + (size_t)(ch * 8) * p.R + r;
+#pragma unroll
+            for (int q4 = 0; q4 < 8; ++q4)
+              dst[(size_t)q4 * p.R] = make_float4(__uint_as_float(ov[4 * q4]), __uint_as_float(ov[4 * q4 + 1]),
+                                                  __uint_as_float(ov[4 * q4 + 2]), __uint_as_float(ov[4 * q4 + 3]));
+          }
+        }
+        if (valid) {
+          partk[(size_t)p.R * D + r] = ref;
+          partk[(size_t)p.R * D + p.R + r] = l_run;
+        }
+        tc_fence_before_sync();
+        if (!ok) break;
+        continue;
+      }
       // merge the F copies of each row (M = max reference, w = 2^(ref - M));
       // copy 0 then normalises and writes a whole segment, or leaves a split
       // one's fp32 partial O [R][D] (relative to M), M [R], L [R]
@@ -826,8 +854,10 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
 // seq_lens, so that after it only the partials are read: one item per output
 // quad (row r, columns 4c4 .. 4c4+3) of every split segment, consecutive
 // threads on consecutive rows of one quad (the [D/4][R] slots make a warp's
-// loads contiguous), with the loads of kTcMergeBatch pieces in flight at
-// once.  In piece order (deterministic):
+// loads contiguous), with the loads of kTcMergeBatch partials in flight at
+// once.  A segment's partials are its pieces' key-split copies (F per piece,
+// F = 4 / 2 / 1 for R <= 32 / 64 / 128), merged in piece-then-copy order
+// (deterministic):
 //   M = max_q m_q,  L = sum_q l_q 2^(m_q - M),  O = sum_q 2^(m_q - M) O_q / L,
 //   lse = (M + log2 L) ln 2.
 // Launched right after the split kernel with programmatic stream
@@ -869,7 +899,9 @@ verify_tc_merge_kernel(const __grid_constant__ AttnParams p) {
     int c_first, n_pieces;
     tc_segment(tp, p, s_prefix, s_cpre, b, h_kv, c_first, n_pieces);
     if (n_pieces <= 1) continue;  // the split kernel wrote the output
-    const float *slot0 = p.partials + (size_t)(c_first + seg) * stride;
+    const int F = p.R <= 32 ? 4 : (p.R <= 64 ? 2 : 1);  // key-split copies per piece
+    const float *slot0 = p.partials + (size_t)(c_first + seg) * F * stride;
+    n_pieces *= F;
     float M = -INFINITY, Ls = 0.f;
     float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
     for (int q0 = 0; q0 < n_pieces; q0 += kTcMergeBatch) {
