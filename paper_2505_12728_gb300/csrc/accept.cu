@@ -58,9 +58,10 @@ struct alignas(16) RowStat {  // a target row, or a run of its chunks (one 16-by
   ff S;            // sum of exp((x - m) / tau); 0 for greedy rows
 };
 
-struct SeqState {
+struct alignas(16) SeqState {  // what the draw needs, in one 16-byte load
   int j;           // first rejected position (k if none)
-  int pad[3];
+  float m;         // row j's largest raw logit
+  ff S;            // row j's sum of exp((x - m) / tau)
 };
 
 struct alignas(16) DrawPart {  // one segment of row j
@@ -161,7 +162,7 @@ __device__ void decide_sequence(const AccParams &p, int b, bool greedy, float ta
     if (tid == 0) {
       if (write) {
         p.num_accepted[b] = j;
-        p.seqs[b].j = j;
+        p.seqs[b] = SeqState{j, s_rm[j], s_rS[j]};
       }
       if (s_j) *s_j = j;
     }
@@ -762,12 +763,14 @@ accept_draw_kernel(const __grid_constant__ AccParams p) {
   const float tau = p.tau[b];
   if (!(tau > 0.0f)) return;  // greedy sequences are complete
   const float u_k = p.u[(size_t)b * (k + 1) + k];
-  grid_dependency_wait();     // j and the row statistics come from the previous kernel
-  const int j = __ldcg(&p.seqs[b].j);
-  const RowStat rs = {__ldcg(&p.rows[(size_t)b * (k + 1) + j].m),
-                      __ldcg(&p.rows[(size_t)b * (k + 1) + j].arg),
-                      ff{__ldcg(&p.rows[(size_t)b * (k + 1) + j].S.hi),
-                         __ldcg(&p.rows[(size_t)b * (k + 1) + j].S.lo)}};
+  grid_dependency_wait();     // j and row j's statistics come from the previous kernel
+  const int4 sq = __ldcg(reinterpret_cast<const int4 *>(p.seqs + b));
+  const int j = sq.x;
+  if (j < 0 || j > k) {       // no decision was written (a timed-out statistics pass)
+    if (c == 0 && threadIdx.x == 0) set_status(p.status, SF_DEVICE_TIMEOUT);
+    return;
+  }
+  const RowStat rs = {__int_as_float(sq.y), 0, ff{__int_as_float(sq.z), __int_as_float(sq.w)}};
   draw_residual(p, b, c, j, rs, tau, u_k);
 }
 
@@ -938,6 +941,8 @@ __device__ void decide_warp(const AccParams &p, int b) {
   const unsigned rejected = __ballot_sync(0xffffffffu, lane < k && !acc);
   const int j = rejected ? __ffs(rejected) - 1 : k;
   const int arg_j = __shfl_sync(0xffffffffu, rarg, j);
+  const float m_j = __shfl_sync(0xffffffffu, rm, j);
+  const ff S_j = ff{__shfl_sync(0xffffffffu, rS.hi, j), __shfl_sync(0xffffffffu, rS.lo, j)};
   if (lane <= k) {
     int v = -1;
     if (lane < j) v = tok;
@@ -946,7 +951,7 @@ __device__ void decide_warp(const AccParams &p, int b) {
   }
   if (lane == 0) {
     p.num_accepted[b] = j;
-    p.seqs[b].j = j;
+    p.seqs[b] = SeqState{j, m_j, S_j};
   }
 }
 

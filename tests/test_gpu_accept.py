@@ -264,3 +264,81 @@ def test_longest_draft_matches_oracle(oracle_mod, V, mode):
     n, toks, ratio = run_accept(inp)
     excluded = compare_accept(ref, n, toks, ratio)
     assert excluded <= 1
+
+
+@pytest.mark.parametrize("V,support", [
+    # V = 40000: 512 tokens per warp, 4096 per CTA of the 16-CTA draw cluster
+    (40000, [0, 511, 512, 4095, 4096, 20479, 20480, 39999]),
+    # V = 152064: 1280 tokens per warp, 10240 per CTA
+    (152064, [0, 1279, 1280, 10239, 10240, 81919, 81920, 152063]),
+    # V % 4 != 0: the draw that searches segment sums after a ticket
+    (40001, [0, 1023, 1024, 8191, 8192, 20480, 39999, 40000]),
+])
+def test_monte_carlo_large_vocabulary_draw(V, support):
+    # The speculative-sampling guarantee at V > 32768 (statistics kernel and
+    # a separate draw): the target has mass only on `support` (its tokens sit
+    # on both sides of the draw's warp and CTA boundaries), the draft on an
+    # overlapping set, so that the residual draw and the bonus draw both
+    # matter.  2^15 trials in 64 launches of 512 sequences.
+    rng = np.random.default_rng(V)
+    k = 2
+    sup = np.array(support)
+    dsup = np.array(sorted(set(support[::2]) | {support[3], support[5]}))
+    logits_rows = np.full((k + 1, V), -np.inf, np.float32)
+    logits_rows[:, sup] = rng.standard_normal((k + 1, len(sup))).astype(np.float32)
+    q_rows = np.zeros((k, V), np.float32)
+    q_rows[:, dsup] = softmax(rng.standard_normal((k, len(dsup))), axis=-1).astype(np.float32)
+    p = softmax(logits_rows.astype(np.float64), axis=-1)
+    Bl, launches = 512, 64
+    logits = torch.from_numpy(logits_rows).cuda().unsqueeze(0).expand(Bl, k + 1, V).contiguous()
+    q = torch.from_numpy(q_rows).cuda().unsqueeze(0).expand(Bl, k, V).contiguous()
+    temp = torch.ones(Bl, dtype=torch.float32, device="cuda")
+    qd = q_rows[:, dsup].astype(np.float64)
+    qc = np.cumsum(qd, axis=-1)
+    ws = sfv.new_workspace(sfv.accept_workspace_size(Bl, k, V))
+    ns, outs = [], []
+    for _ in range(launches):
+        toks = np.stack([dsup[np.minimum(np.searchsorted(qc[i], rng.random(Bl) * qc[i, -1],
+                                                         side="right"), len(dsup) - 1)]
+                         for i in range(k)], axis=1).astype(np.int32)
+        u = rng.random((Bl, k + 1), dtype=np.float32)
+        n, o, _ = sfv.accept(logits, q, torch.from_numpy(toks).cuda(), torch.from_numpy(u).cuda(),
+                             temp, workspace=ws)
+        ns.append(n)
+        outs.append(o)
+    assert sfv.read_device_status(ws) == 0
+    n = torch.cat(ns).cpu().numpy()
+    out = torch.cat(outs).cpu().numpy()
+    trials = n.shape[0]
+    alpha = 1e-4
+    for i in range(k + 1):
+        sel = n >= i
+        emitted = out[sel, i]
+        assert np.isin(emitted, sup).all(), np.setdiff1d(emitted, sup)
+        obs = np.array([(emitted == t).sum() for t in sup])
+        assert chisquare(obs, p[i, sup] * sel.sum()).pvalue > alpha, (i, obs, p[i, sup] * sel.sum())
+    beta = np.minimum(p[:k], q_rows.astype(np.float64)).sum(axis=-1)
+    surv = np.concatenate([[1.0], np.cumprod(beta)])
+    law = np.append(surv[:-1] - surv[1:], surv[-1])
+    obs = np.bincount(n, minlength=k + 1)
+    assert chisquare(obs, law * trials).pvalue > alpha, (obs, law * trials)
+
+
+@pytest.mark.parametrize("V", [40000, 40001, 152064])
+def test_residual_without_mass_draws_from_the_target(oracle_mod, V):
+    # q = 1.001 p everywhere: the residual max(0, p - q) is exactly zero, and
+    # u_0 = 0.9995 > p/q rejects the first draft (by a relative margin of
+    # 5e-4), so the token comes from p_0 itself on both sides (logits with a
+    # wide spread, so that the draw's CDF steps are large against the
+    # oracle's 1e-6 margin)
+    rng = np.random.default_rng(V + 1)
+    B, k = 8, 2
+    logits = (6.0 * rng.standard_normal((B, k + 1, V))).astype(np.float32)
+    p = softmax(logits.astype(np.float64), axis=-1)
+    q = (1.001 * p[:, :k]).astype(np.float32)
+    tokens = np.argmax(q, axis=-1).astype(np.int32)
+    u = rng.random((B, k + 1), dtype=np.float32)
+    u[:, 0] = 0.9995
+    inp = AcceptInputs(logits, q, tokens, u, np.ones(B, np.float32))
+    ref, n, toks = _check(oracle_mod, inp, max_excluded_frac=0.0)
+    assert (n == 0).all()
