@@ -140,9 +140,11 @@ def attention_bytes_per_layer(wl, seq_lens) -> int:
 
 
 def accept_bytes(wl, mode_sampling_rows: int) -> int:
-    """Algorithmic bytes of acceptance: all (k+1) logits rows once, plus one
-    row of logits and one of q per sampled sequence for the draw."""
-    return wl.B * (wl.k + 1) * wl.V * 4 + mode_sampling_rows * wl.V * 4 * 2
+    """Algorithmic bytes of acceptance: all (k+1) logits rows once, plus row j
+    of q for each sampled sequence's draw.  The draw's second read of row j
+    of the logits (usually still in L2) is implementation overhead, reported
+    separately (accept_reread_bytes)."""
+    return wl.B * (wl.k + 1) * wl.V * 4 + mode_sampling_rows * wl.V * 4
 
 
 # Sources whose code (comments and layout removed) a committed ncu summary
@@ -575,13 +577,14 @@ def l2_bytes():
         return 129 << 20
 
 
-def time_workload(name, dev, stream, capture, peak, reps=20):
+def time_workload(name, dev, stream, capture, peak, min_calls=200):
     """Attention and acceptance of one more workload, each replayed from a
     CUDA graph that rotates over enough distinct inputs (independent layers
     of KV; copies of the acceptance inputs) to exceed twice the L2, so every
-    call streams from HBM.  Reports per-call device times (CUDA events on the
-    launching stream), algorithmic GB/s and the fraction of the measured copy
-    bandwidth."""
+    call streams from HBM, for at least min_calls calls after warm-up.
+    Reports per-call device times (CUDA events on the launching stream: the
+    mean, and p10 / median / p90 over the replays), algorithmic GB/s and the
+    fractions of the measured copy bandwidth and of the nominal 8 TB/s."""
     import torch
     from paper_2505_12728_gb300 import specflash_verify as sfv
     from paper_2505_12728_gb300.workloads import make_accept_inputs, workload
@@ -605,21 +608,26 @@ def time_workload(name, dev, stream, capture, peak, reps=20):
                                  lse=e, workspace=ws, stream=stream)
 
     def timed(fn, calls):
+        """Mean per-call µs over the replays, and {p10, median, p90} of the
+        per-replay means (an event between replays)."""
         fn()
         g = capture(fn)
         for _ in range(3):
             g.replay()
-        a = torch.cuda.Event(enable_timing=True)
-        b = torch.cuda.Event(enable_timing=True)
+        reps = max(20, -(-min_calls // calls))
+        ev = [torch.cuda.Event(enable_timing=True) for _ in range(reps + 1)]
         torch.cuda.synchronize()
-        a.record(stream)
-        for _ in range(reps):
+        ev[0].record(stream)
+        for i in range(reps):
             g.replay()
-        b.record(stream)
+            ev[i + 1].record(stream)
         torch.cuda.synchronize()
-        return a.elapsed_time(b) * 1e3 / (calls * reps)
+        per = np.array([ev[i].elapsed_time(ev[i + 1]) * 1e3 / calls for i in range(reps)])
+        dist = {"p10": float(np.percentile(per, 10)), "median": float(np.median(per)),
+                "p90": float(np.percentile(per, 90)), "calls": calls * reps}
+        return ev[0].elapsed_time(ev[reps]) * 1e3 / (calls * reps), dist
 
-    att_us = timed(attn_all, n_layers)
+    att_us, att_dist = timed(attn_all, n_layers)
     att_status = sfv.read_device_status(ws)
     finite = all(bool(torch.isfinite(e).all().item()) for e in lses)
     del layers, outs
@@ -640,7 +648,7 @@ def time_workload(name, dev, stream, capture, peak, reps=20):
             sfv.accept(*c, num_accepted=n_acc, out_tokens=toks, accept_ratio=ratio,
                        workspace=ws_a, stream=stream)
 
-    acc_us = timed(acc_all, n_copies)
+    acc_us, acc_dist = timed(acc_all, n_copies)
     sampling_rows = int(np.sum(acc.temperature > 0))
     acc_bytes = accept_bytes(wl, sampling_rows)
     # the data-dependent minimum: the logits rows 0..min(j, k) of each
@@ -655,16 +663,20 @@ def time_workload(name, dev, stream, capture, peak, reps=20):
             "attention_kernel": attention_kernel(wl),
             "attention_launches_per_call": sfv.verify_attention_kernel_launches(
                 wl.B, wl.rows, wl.H_q, wl.H_kv, wl.d, max_pages),
-            "attention_us": att_us, "attention_algorithmic_bytes": bytes_layer,
-            "kv_gbs": kv_gbs, "frac": kv_gbs / peak,
+            "attention_us": att_us, "attention_us_distribution": att_dist,
+            "attention_algorithmic_bytes": bytes_layer,
+            "kv_gbs": kv_gbs, "frac": kv_gbs / peak, "frac_of_nominal_8tbs": kv_gbs / 8000.0,
             "layers_rotated": n_layers, "attention_finite": finite,
             "accept_kernels": (["accept_cluster_kernel"] if sfv.accept_kernel_launches(
                 wl.B, wl.k, wl.V) == 1 else ["accept_chunks_kernel", "accept_draw_kernel"]),
-            "accept_us": acc_us, "accept_algorithmic_bytes": acc_bytes, "accept_gbs": acc_gbs,
+            "accept_us": acc_us, "accept_us_distribution": acc_dist,
+            "accept_algorithmic_bytes": acc_bytes, "accept_gbs": acc_gbs,
+            "accept_reread_bytes": sampling_rows * wl.V * 4,
             "accept_min_bytes": acc_min_bytes, "accept_min_gbs": acc_min_bytes / (acc_us * 1e-6) / 1e9,
             "merge_partial_bytes": tc_merge_partial_bytes(
                 wl, seq_np, torch.cuda.get_device_properties(dev).multi_processor_count),
-            "accept_frac": acc_gbs / peak, "accept_input_copies_rotated": n_copies,
+            "accept_frac": acc_gbs / peak, "accept_frac_of_nominal_8tbs": acc_gbs / 8000.0,
+            "accept_input_copies_rotated": n_copies,
             "mean_accepted": float(n_acc.float().mean().item()),
             "device_status": att_status | sfv.read_device_status(ws_a)}
 
