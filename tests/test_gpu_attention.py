@@ -250,6 +250,9 @@ def test_kernel_launch_counts_follow_the_rows_per_kv_head():
     (1, 16, 8, 1, 128, (20000, 20000)),  # one 128-row segment over every CTA
     (1, 16, 8, 1, 64, (20000, 20000)),
     (1, 8, 28, 4, 128, (30000, 30000)),  # four 56-row segments of ~38 pieces each
+    (1, 4, 28, 4, 128, (30000, 30000)),  # 28 rows (four key-split copies): ~152
+                                         # partials per segment and row
+    (2, 3, 16, 2, 64, (12000, 12000)),   # 24 rows, head_dim 64, four copies
     (40, 8, 28, 4, 128, (500, 3000)),    # 160 segments > 152 CTAs: balanced partition,
                                          # a CTA's first and last pieces split
 ])
