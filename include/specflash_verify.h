@@ -98,6 +98,14 @@ int sf_workspace_init(void *workspace, size_t bytes, cudaStream_t stream);
  * *status_out holds the SF_DEVICE_* bits; returns SF_OK or SF_ERR_CUDA. */
 int sf_read_device_status(const void *workspace, uint32_t *status_out);
 
+/* Self-test of the bounded waits (diagnostics): launches one CTA whose      */
+/* thread waits on an mbarrier that nothing completes.  The wait gives up    */
+/* after about one second (the budget of every wait in these kernels) and    */
+/* sets SF_DEVICE_TIMEOUT in the status word at the start of `workspace`     */
+/* (>= 4 bytes, 4-byte aligned); the context stays usable.  Returns SF_OK or */
+/* SF_ERR_WORKSPACE / SF_ERR_CUDA; asynchronous on `stream`.                 */
+int sf_selftest_bounded_wait(void *workspace, size_t workspace_bytes, cudaStream_t stream);
+
 /* ------------------------------------------------------------------------ */
 /* Verification attention (Sec. 3.1: the K candidates' probabilities come  */
 /* from one parallel forward pass of the target model; the verify costs     */

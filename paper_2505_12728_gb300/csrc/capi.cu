@@ -6,6 +6,7 @@
 #include <cstring>
 #include <mutex>
 
+#include "sf_device.cuh"
 #include "sf_host.h"
 
 namespace sf {
@@ -81,6 +82,19 @@ int encode_tensor_map_bf16(CUtensorMap *map, const void *base, int rank, const u
   return SF_OK;
 }
 
+// Self-test of the bounded wait every kernel uses: one thread waits for
+// phase 0 of an mbarrier that nobody arrives at.  The wait gives up after
+// kWaitBudgetNs and the kernel records SF_DEVICE_TIMEOUT, as the kernels do
+// when a copy or a peer never completes.
+__global__ void selftest_wait_kernel(uint32_t *status) {
+  __shared__ alignas(8) uint64_t bar;
+  if (threadIdx.x == 0) {
+    mbar_init(smem_addr(&bar), 1);
+    fence_mbar_init();
+    if (!mbar_wait_bounded(smem_addr(&bar), 0u)) set_status(status, SF_DEVICE_TIMEOUT);
+  }
+}
+
 }  // namespace sf
 
 extern "C" {
@@ -105,6 +119,16 @@ int sf_workspace_init(void *workspace, size_t bytes, cudaStream_t stream) {
   if (!workspace || bytes == 0) return sf::fail(SF_ERR_INVALID_ARG, "workspace is NULL or empty");
   cudaError_t e = cudaMemsetAsync(workspace, 0, bytes, stream);
   if (e != cudaSuccess) return sf::fail(SF_ERR_CUDA, "cudaMemsetAsync: %s", cudaGetErrorString(e));
+  return SF_OK;
+}
+
+int sf_selftest_bounded_wait(void *workspace, size_t workspace_bytes, cudaStream_t stream) {
+  sf::clear_error();
+  if (!workspace || workspace_bytes < sizeof(uint32_t) || !sf::aligned(workspace, 4))
+    return sf::fail(SF_ERR_WORKSPACE, "workspace must hold a 4-byte aligned status word");
+  sf::selftest_wait_kernel<<<1, 32, 0, stream>>>(static_cast<uint32_t *>(workspace));
+  const cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return sf::fail(SF_ERR_CUDA, "self-test launch: %s", cudaGetErrorString(e));
   return SF_OK;
 }
 

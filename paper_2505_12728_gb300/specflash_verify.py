@@ -27,7 +27,8 @@ PAGE_SIZE = 16
 
 EXPORTED_SYMBOLS = (
     "sf_status_string", "sf_last_error", "sf_version", "sf_workspace_init",
-    "sf_read_device_status", "sf_verify_attention_workspace_size", "sf_verify_attention",
+    "sf_read_device_status", "sf_selftest_bounded_wait",
+    "sf_verify_attention_workspace_size", "sf_verify_attention",
     "sf_verify_attention_noalloc", "sf_verify_attention_kernel_launches",
     "sf_accept_workspace_size", "sf_accept", "sf_accept_kernel_launches",
     "sf_kv_commit_workspace_size", "sf_kv_commit",
@@ -74,6 +75,8 @@ def load_library(path: str | None = None):
         lib.sf_workspace_init.restype = I
         lib.sf_read_device_status.argtypes = [P, ctypes.POINTER(ctypes.c_uint32)]
         lib.sf_read_device_status.restype = I
+        lib.sf_selftest_bounded_wait.argtypes = [P, S, P]
+        lib.sf_selftest_bounded_wait.restype = I
         lib.sf_verify_attention_workspace_size.argtypes = [I, I, I, I, I, I, I, I]
         lib.sf_verify_attention_workspace_size.restype = S
         lib.sf_verify_attention.argtypes = [P, P, P, P, P, I, I, I, I, I, I, I, I, F, I, P, P, P,
@@ -203,6 +206,15 @@ def read_device_status(workspace: torch.Tensor) -> int:
     v = ctypes.c_uint32(0)
     _check(load_library().sf_read_device_status(_ptr(workspace), ctypes.byref(v)))
     return int(v.value)
+
+
+def selftest_bounded_wait(workspace: torch.Tensor, stream=None) -> None:
+    """sf_selftest_bounded_wait: a wait that nothing completes gives up after
+    about a second and sets SF_DEVICE_TIMEOUT in the workspace's status word
+    (read it with read_device_status)."""
+    _need_workspace(workspace)
+    _check(load_library().sf_selftest_bounded_wait(_ptr(workspace), workspace.numel(),
+                                                   _stream_handle(stream)))
 
 
 # --------------------------------------------------------------------------- #

@@ -296,3 +296,19 @@ def test_outputs_beyond_four_are_judged_against_their_bf16_rounding(oracle_mod):
     out, lse = run_attention(case, num_splits=7)
     assert np.abs(out - ref_out).max() > 1e-2           # the bf16 format alone
     assert_attention_close(out, lse, ref_out, ref_lse)  # within 1e-2 beyond it
+
+
+def test_a_wait_that_runs_out_reports_a_timeout_and_the_context_stays_usable(oracle_mod):
+    # The bounded wait the kernels use, on an mbarrier nothing completes:
+    # after ~1 s it gives up and sets SF_DEVICE_TIMEOUT; no fault, no hang.
+    import time
+    ws = sfv.new_workspace(256)
+    t0 = time.time()
+    sfv.selftest_bounded_wait(ws)
+    assert sfv.read_device_status(ws) == sfv.SF_DEVICE_TIMEOUT
+    assert 0.5 < time.time() - t0 < 30
+    # the context still runs both kernels correctly
+    case = make_attention_case(2, 8, 28, 4, 128, [300, 1000], seed=85)
+    out, lse = run_attention(case)
+    ref_out, ref_lse = oracle_attention(oracle_mod, case)
+    assert_attention_close(out, lse, ref_out, ref_lse)
