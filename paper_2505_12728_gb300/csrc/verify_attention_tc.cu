@@ -57,10 +57,12 @@
 //  * A piece that covers a whole segment writes bf16 out and the LSE; a
 //    split segment's pieces write fp32 partials to the workspace, one per
 //    key-split copy (O as [D/4][R] float4, so that a warp's stores are
-//    contiguous), which
-//    verify_tc_merge_kernel combines across the whole GPU right after this
-//    kernel (one CTA merging a segment's ~250 KB of partials alone took
-//    longer than the whole split phase).
+//    contiguous), which verify_tc_merge_kernel combines across the whole
+//    GPU right after this kernel.  As a separate kernel the merge also lets
+//    the next call's CTAs take the SMs this grid leaves, and run their
+//    prologue and first copies while it merges; one CTA merging a
+//    segment's partials alone, or every CTA merging after a grid-wide
+//    barrier, kept the SMs busy and exposed that prologue.
 //  * K/V copies run before griddepcontrol.wait only for tiles that lie
 //    wholly in the prefix; tiles holding draft positions
 //    (which the previous kernel on the stream may have just written) are
