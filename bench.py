@@ -883,55 +883,75 @@ def run_ours(args):
         others[name] = time_workload(name, dev, stream, capture, peak_gbs)
         torch.cuda.empty_cache()
 
-    # ---- end to end through host buffers: the step's inputs are packed in
-    # one pinned staging buffer (one host-to-device copy per step) and its
-    # results in one device buffer (one device-to-host copy) ----
+    # ---- end to end through host buffers: each step's inputs are packed in
+    # one pinned staging buffer and copied to the device in one host-to-device
+    # copy, and its results come back in one device-to-host copy.  The copy
+    # of step s + 1's inputs runs on a side stream while step s computes (two
+    # pinned and two device staging buffers, alternating), and each step
+    # joins it at its end ----
     inputs = [att.q.view(np.int16), acc.target_logits, acc.draft_probs, acc.draft_tokens,
               acc.uniforms, acc.temperature]
     offs, total = [], 0
     for a in inputs:
         offs.append(total)
         total += (a.nbytes + 255) // 256 * 256
-    h_stage = torch.empty(total, dtype=torch.uint8).pin_memory()
-    for a, o in zip(inputs, offs):
-        h_stage[o:o + a.nbytes].copy_(torch.from_numpy(np.ascontiguousarray(a).view(np.uint8).reshape(-1)))
-    d_stage = torch.empty(total, dtype=torch.uint8, device=dev)
+    h_stages = [torch.empty(total, dtype=torch.uint8).pin_memory() for _ in range(2)]
+    for h_stage in h_stages:
+        for a, o in zip(inputs, offs):
+            h_stage[o:o + a.nbytes].copy_(torch.from_numpy(np.ascontiguousarray(a).view(np.uint8).reshape(-1)))
+    d_stages = [torch.empty(total, dtype=torch.uint8, device=dev) for _ in range(2)]
 
-    def staged(i, dtype, shape):
+    def staged(d_stage, i, dtype, shape):
         n = inputs[i].nbytes
         return d_stage[offs[i]:offs[i] + n].view(dtype).view(shape)
 
-    d_q = staged(0, torch.bfloat16, tuple(q.shape))
-    d_logits = staged(1, torch.float32, tuple(logits.shape))
-    d_qprob = staged(2, torch.float32, tuple(qprob.shape))
-    d_toks = staged(3, torch.int32, tuple(toks.shape))
-    d_uni = staged(4, torch.float32, tuple(uni.shape))
-    d_temp = staged(5, torch.float32, tuple(temp.shape))
+    views = [(staged(d, 0, torch.bfloat16, tuple(q.shape)), staged(d, 1, torch.float32, tuple(logits.shape)),
+              staged(d, 2, torch.float32, tuple(qprob.shape)), staged(d, 3, torch.int32, tuple(toks.shape)),
+              staged(d, 4, torch.float32, tuple(uni.shape)), staged(d, 5, torch.float32, tuple(temp.shape)))
+             for d in d_stages]
+    copy_stream = torch.cuda.Stream(device=dev)
     d_res = torch.empty(wl.B * (wl.k + 2), dtype=torch.int32, device=dev)
     e_n, e_out = d_res[:wl.B], d_res[wl.B:].view(wl.B, wl.k + 1)
     h_res = torch.empty(wl.B * (wl.k + 2), dtype=torch.int32).pin_memory()
     h_n, h_out = h_res[:wl.B], h_res[wl.B:].view(wl.B, wl.k + 1)
-    h2d = h_stage.numel()  # the packed inputs (each padded to 256 bytes)
+    h2d = h_stages[0].numel()  # one step's packed inputs (each padded to 256 bytes)
     d2h = h_res.numel() * 4
 
-    def e2e_step():
-        d_stage.copy_(h_stage, non_blocking=True)
+    def e2e_step(par):
+        # this step's inputs are in d_stages[par]; the next step's are copied
+        # into the other buffer (free once the previous step is done) meanwhile
+        copy_stream.wait_stream(stream)
+        with torch.cuda.stream(copy_stream):
+            d_stages[1 - par].copy_(h_stages[1 - par], non_blocking=True)
+        d_q, d_logits, d_qprob, d_toks, d_uni, d_temp = views[par]
         attention_layers(d_q)
         sfv.accept(d_logits, d_qprob, d_toks, d_uni, d_temp, num_accepted=e_n, out_tokens=e_out,
                    accept_ratio=ratio, workspace=ws_acc, stream=stream)
         h_res.copy_(d_res, non_blocking=True)
+        stream.wait_stream(copy_stream)
 
-    for _ in range(args.warmup):
-        e2e_step()
+    d_stages[0].copy_(h_stages[0], non_blocking=True)  # the first step's inputs
+    for i in range(args.warmup):
+        e2e_step(i % 2)
     torch.cuda.synchronize()
-    run_e2e = capture(e2e_step).replay if use_graph else e2e_step
+    if use_graph:
+        g_par = [capture(lambda: e2e_step(0)), capture(lambda: e2e_step(1))]
+        run_e2e = lambda i: g_par[i % 2].replay()
+    else:
+        run_e2e = e2e_step
+    # the step counter continues across warm-up and the timed steps, so that
+    # every step reads the buffer the previous one filled
+    step_i = 0
+    d_stages[0].copy_(h_stages[0], non_blocking=True)
     for _ in range(args.warmup):
-        run_e2e()
+        run_e2e(step_i % 2)
+        step_i += 1
     torch.cuda.synchronize()
     barrier(world)
     e0.record(stream)
     for _ in range(args.steps):
-        run_e2e()
+        run_e2e(step_i % 2)
+        step_i += 1
     e1.record(stream)
     torch.cuda.synchronize()
     barrier(world)
