@@ -340,31 +340,69 @@ def run_reference(args):
     wl = workload(args.workload, **({"layers": args.layers} if args.layers else {}))
     att = make_attention_inputs(wl, layers=min(wl.layers, 2))
     acc = make_accept_inputs(wl)
-    def full_step():
-        # every layer of the step (the inputs of two generated layers, used in
-        # turn: the oracle's time does not depend on the values), then the
-        # acceptance
-        for l in range(wl.layers):
-            oracle.verify_attention(att.q[l % att.layers], att.k_cache[l % att.layers],
-                                    att.v_cache[l % att.layers], att.block_table[l % att.layers],
-                                    att.seq_lens, H_kv=att.H_kv)
+
+    def layer(l):
+        # the inputs of two generated layers, used in turn (the oracle's time
+        # does not depend on the values)
+        oracle.verify_attention(att.q[l % att.layers], att.k_cache[l % att.layers],
+                                att.v_cache[l % att.layers], att.block_table[l % att.layers],
+                                att.seq_lens, H_kv=att.H_kv)
+
+    def accept():
         oracle.accept(acc.target_logits, acc.draft_probs, acc.draft_tokens, acc.uniforms,
                       acc.temperature)
 
+    # Each step is a bounded sample of the workload: as many of its layers as
+    # let all W + K steps end within the wall-clock budget (all of them when
+    # they fit), then the acceptance.  Layer and acceptance times are
+    # measured apart, so that a sampled step's attention time can be scaled
+    # to the workload's layer count.
+    t = time.perf_counter()
+    layer(0)
+    t_layer = time.perf_counter() - t
+    t = time.perf_counter()
+    accept()
+    t_acc = time.perf_counter() - t
+    n_steps = args.warmup + args.steps
+    per_step = args.reference_budget / n_steps
+    n_layers = int(min(wl.layers, max(1, (per_step - t_acc) // max(t_layer, 1e-9))))
+
+    def step():
+        t = time.perf_counter()
+        for l in range(n_layers):
+            layer(l)
+        t_att = time.perf_counter() - t
+        accept()
+        return t_att
+
     for _ in range(args.warmup):
-        full_step()
+        step()
+    att_s = 0.0
     t0 = time.perf_counter()
     for _ in range(args.steps):
-        full_step()
+        att_s += step()
     step_s = (time.perf_counter() - t0) / args.steps
-    value = wl.B * wl.k / step_s
-    sample = (f"each step: the fp64 C oracle on all {wl.layers} attention layers plus the "
-              f"acceptance of the {wl.name} workload, measured (no extrapolation)")
+    att_step_s = att_s / args.steps
+    # the workload's full step: the attention of all its layers (scaled from
+    # the sampled ones when fewer ran) plus the measured acceptance
+    full_step_s = att_step_s * wl.layers / n_layers + (step_s - att_step_s)
+    value = wl.B * wl.k / full_step_s
+    if n_layers == wl.layers:
+        sample = (f"each step: the fp64 C oracle on all {wl.layers} attention layers plus the "
+                  f"acceptance of the {wl.name} workload, measured (no extrapolation)")
+    else:
+        sample = (f"each step: the fp64 C oracle on {n_layers} of the {wl.name} workload's "
+                  f"{wl.layers} attention layers plus its acceptance (so that {n_steps} steps "
+                  f"fit {args.reference_budget:.0f} s); ms_per_step is that measured step, and "
+                  f"value is draft tokens per full step with the attention time scaled by "
+                  f"{wl.layers}/{n_layers}")
     line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT,
             "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": step_s * 1e3, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "f64", "data": "synthetic",
             "config": workload_config(wl, att.seq_lens),
+            "layers_per_step": n_layers,
+            "ms_per_full_step": full_step_s * 1e3,
             "cpu_baseline": {"value": value, "unit": UNIT, "cores": oracle_cores(),
                              "kind": "oracle", "sample": sample},
             "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0,
@@ -1032,6 +1070,9 @@ def main(argv=None):
     ap.add_argument("--cpu-budget", type=float, default=12.0,
                     help="seconds of oracle work for the cpu_baseline sample")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--reference-budget", type=float, default=150.0,
+                    help="--impl reference: wall-clock seconds for all warm-up and timed steps; "
+                         "each step runs as many of the workload's layers as fit")
     ap.add_argument("--no-draft-tail", action="store_true",
                     help="skip the draft-side and LM-head timings (draft tail, visual compressor, "
                          "fused target LM head + acceptance)")

@@ -56,6 +56,22 @@ def test_reference_arm_prints_one_json_line():
     assert d["config"]["workload"] == "tiny"
 
 
+def test_reference_arm_samples_layers_to_fit_its_budget():
+    # a budget far below one full step: each step runs one of the four
+    # layers, ms_per_step is that step, and the full step is scaled from it
+    env = dict(os.environ, OMP_NUM_THREADS="2")
+    r = subprocess.run([sys.executable, "bench.py", "--impl", "reference", "--workload", "tiny",
+                        "--layers", "4", "--steps", "2", "--warmup", "3",
+                        "--reference-budget", "0.001"], cwd=ROOT, env=env,
+                       capture_output=True, text=True, timeout=600)
+    assert r.returncode == 0, r.stderr
+    d = json.loads(r.stdout.strip().splitlines()[-1])
+    assert d["layers_per_step"] == 1 and d["steps"] == 2 and d["warmup"] == 3
+    assert "1 of the tiny workload's 4 attention layers" in d["cpu_baseline"]["sample"]
+    assert d["ms_per_full_step"] > d["ms_per_step"]
+    assert abs(d["value"] - d["cpu_baseline"]["value"]) == 0
+
+
 def test_reference_arm_is_silent_on_other_ranks():
     env = dict(os.environ, RANK="1", WORLD_SIZE="2", LOCAL_RANK="1")
     r = subprocess.run([sys.executable, "bench.py", "--impl", "reference", "--steps", "1"],
