@@ -449,14 +449,6 @@ __device__ __forceinline__ void tmem_wait_st() {
   asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
 }
 
-// Load with acquire semantics at GPU scope (pairs with a release or a
-// __threadfence() before an atomic in another CTA).
-__device__ __forceinline__ uint32_t ld_acquire_gpu(const uint32_t *p) {
-  uint32_t v;
-  asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
-  return v;
-}
-
 // Atomic add with acquire-release semantics at GPU scope.  After a CTA
 // barrier, one thread's add releases the writes of the whole CTA, and its
 // result acquires the writes that earlier adds released (a barrier after it
